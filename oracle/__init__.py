@@ -1,0 +1,229 @@
+"""CPU oracle for the DynamicPTQ quantized linear layer (ctypes wrapper over dptq_oracle.c).
+
+TEST INFRASTRUCTURE ONLY: the test suite, ``__graft_entry__.smoke()`` and the CPU-baseline
+leg of ``bench.py`` may use it; the product path (``paper_2606_12487_gb300``) never does.
+It shares no code with the CUDA library.  See ``dptq_oracle.c`` for the definitions and the
+paper passages each function follows (Section 2 Eqs. 2-5, Section 4.2, Section 3.1 Eqs. 8-11).
+
+Parity status: every exported function is pinned by tests under ``tests/test_oracle_*.py``
+against closed forms, textbook constructions and library routines.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "dptq_oracle.c")
+_LIB = os.path.join(_HERE, "_build", "libdptq_oracle.so")
+_lock = threading.Lock()
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle with the host C compiler (plain C11, no fast-math)."""
+    os.makedirs(os.path.dirname(_LIB), exist_ok=True)
+    if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
+        tmp = _LIB + f".tmp{os.getpid()}"
+        subprocess.check_call(
+            ["cc", "-O2", "-std=c11", "-ffp-contract=off", "-fno-fast-math", "-fPIC", "-shared",
+             _SRC, "-o", tmp, "-lm"])
+        os.replace(tmp, _LIB)
+    return _LIB
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is None:
+            lib = ctypes.CDLL(build())
+            P = ctypes.c_void_p
+            I = ctypes.c_int
+            lib.orc_half_to_double.argtypes = [ctypes.c_uint16]
+            lib.orc_half_to_double.restype = ctypes.c_double
+            lib.orc_float_to_half.argtypes = [ctypes.c_float]
+            lib.orc_float_to_half.restype = ctypes.c_uint16
+            lib.orc_hadamard_entry.argtypes = [I, I]
+            lib.orc_hadamard_entry.restype = I
+            lib.orc_block_layout.argtypes = [I, I, P, P]
+            lib.orc_block_layout.restype = I
+            lib.orc_rotate_row_f64.argtypes = [P, P, I, I]
+            lib.orc_rotate_row_f64.restype = I
+            lib.orc_rotate_f16.argtypes = [P, P, I, I, I]
+            lib.orc_rotate_f16.restype = I
+            lib.orc_quant_rows.argtypes = [P, I, I, I, P, P]
+            lib.orc_quant_rows.restype = I
+            lib.orc_rotate_quant_act.argtypes = [P, I, I, I, I, P, P]
+            lib.orc_rotate_quant_act.restype = I
+            lib.orc_pack_weights.argtypes = [P, I, I, I, P, P]
+            lib.orc_pack_weights.restype = I
+            lib.orc_gemm_i32.argtypes = [P, P, I, I, I, P]
+            lib.orc_gemm_i32.restype = I
+            lib.orc_epilogue.argtypes = [P, P, P, I, I, P]
+            lib.orc_epilogue.restype = None
+            lib.orc_qlinear.argtypes = [P, I, I, I, I, P, P, I, P, P, P, P]
+            lib.orc_qlinear.restype = I
+            lib.orc_pack_nibbles.argtypes = [P, I, I, P]
+            lib.orc_pack_nibbles.restype = None
+            lib.orc_unpack_nibbles.argtypes = [P, I, I, P]
+            lib.orc_unpack_nibbles.restype = None
+            lib.orc_residual_stats.argtypes = [P, P, I, I, I, ctypes.c_double, P, P]
+            lib.orc_residual_stats.restype = I
+            _lib = lib
+    return _lib
+
+
+def _p(a: np.ndarray):
+    assert a.flags["C_CONTIGUOUS"]
+    return a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _as_half_bits(x) -> np.ndarray:
+    x = np.ascontiguousarray(x)
+    if x.dtype == np.float16:
+        return x.view(np.uint16)
+    assert x.dtype == np.uint16, x.dtype
+    return x
+
+
+# ---------------------------------------------------------------------------------------
+def half_to_double(bits: int) -> float:
+    return _load().orc_half_to_double(int(bits))
+
+
+def float_to_half(v: float) -> int:
+    return int(_load().orc_float_to_half(float(v)))
+
+
+def hadamard_entry(i: int, j: int) -> int:
+    return int(_load().orc_hadamard_entry(i, j))
+
+
+def block_layout(K: int, B: int):
+    q = ctypes.c_int(0)
+    r = ctypes.c_int(0)
+    ok = _load().orc_block_layout(K, B, ctypes.byref(q), ctypes.byref(r))
+    return (q.value, r.value) if ok else None
+
+
+def rotate_row_f64(x: np.ndarray, B: int) -> np.ndarray:
+    x = np.ascontiguousarray(x, dtype=np.float64)
+    y = np.empty_like(x)
+    if not _load().orc_rotate_row_f64(_p(x), _p(y), x.shape[0], B):
+        raise ValueError("bad block layout")
+    return y
+
+
+def rotate(x_f16: np.ndarray, B: int) -> np.ndarray:
+    """fp16 [M, K] -> fp32 [M, K]: x R with R = blockdiag(H/sqrt(block)) (Eq. 4)."""
+    xb = _as_half_bits(x_f16)
+    M, K = xb.shape
+    y = np.empty((M, K), dtype=np.float32)
+    if not _load().orc_rotate_f16(_p(xb), _p(y), M, K, B):
+        raise ValueError("bad block layout")
+    return y
+
+
+def quant_rows(y: np.ndarray, bits: int):
+    """Per-token symmetric quantizer (Eq. 2, Section 4.2): returns (codes int8, scales fp32)."""
+    y = np.ascontiguousarray(y, dtype=np.float32)
+    M, K = y.shape
+    c = np.empty((M, K), dtype=np.int8)
+    s = np.empty((M,), dtype=np.float32)
+    if not _load().orc_quant_rows(_p(y), M, K, bits, _p(c), _p(s)):
+        raise ValueError("bits must be 4 or 8")
+    return c, s
+
+
+def rotate_quant_act(x_f16: np.ndarray, B: int, bits: int):
+    xb = _as_half_bits(x_f16)
+    M, K = xb.shape
+    c = np.empty((M, K), dtype=np.int8)
+    s = np.empty((M,), dtype=np.float32)
+    if not _load().orc_rotate_quant_act(_p(xb), M, K, B, bits, _p(c), _p(s)):
+        raise ValueError("bad shape or bits")
+    return c, s
+
+
+def pack_weights(W_f16: np.ndarray, B: int):
+    """RTN int4 per-channel symmetric weights with R folded in (Eq. 5): (q int8 [N,K], s_w fp32 [N])."""
+    wb = _as_half_bits(W_f16)
+    N, K = wb.shape
+    q = np.empty((N, K), dtype=np.int8)
+    s = np.empty((N,), dtype=np.float32)
+    if not _load().orc_pack_weights(_p(wb), N, K, B, _p(q), _p(s)):
+        raise ValueError("bad shape")
+    return q, s
+
+
+def gemm_i32(a: np.ndarray, w: np.ndarray) -> np.ndarray:
+    a = np.ascontiguousarray(a, dtype=np.int8)
+    w = np.ascontiguousarray(w, dtype=np.int8)
+    M, K = a.shape
+    N, K2 = w.shape
+    assert K == K2
+    acc = np.empty((M, N), dtype=np.int32)
+    if not _load().orc_gemm_i32(_p(a), _p(w), M, N, K, _p(acc)):
+        raise OverflowError("accumulator leaves int32")
+    return acc
+
+
+def epilogue(acc: np.ndarray, sa: np.ndarray, sw: np.ndarray) -> np.ndarray:
+    acc = np.ascontiguousarray(acc, dtype=np.int32)
+    sa = np.ascontiguousarray(sa, dtype=np.float32)
+    sw = np.ascontiguousarray(sw, dtype=np.float32)
+    M, N = acc.shape
+    out = np.empty((M, N), dtype=np.uint16)
+    _load().orc_epilogue(_p(acc), _p(sa), _p(sw), M, N, _p(out))
+    return out.view(np.float16)
+
+
+def qlinear(x_f16: np.ndarray, B: int, bits: int, q: np.ndarray, sw: np.ndarray):
+    """Whole layer: returns dict(out fp16 [M,N], acc int32, codes int8, sa fp32)."""
+    xb = _as_half_bits(x_f16)
+    M, K = xb.shape
+    q = np.ascontiguousarray(q, dtype=np.int8)
+    sw = np.ascontiguousarray(sw, dtype=np.float32)
+    N = q.shape[0]
+    out = np.empty((M, N), dtype=np.uint16)
+    acc = np.empty((M, N), dtype=np.int32)
+    codes = np.empty((M, K), dtype=np.int8)
+    sa = np.empty((M,), dtype=np.float32)
+    if not _load().orc_qlinear(_p(xb), M, K, B, bits, _p(q), _p(sw), N, _p(out), _p(acc),
+                               _p(codes), _p(sa)):
+        raise ValueError("bad shape, bits or int32 overflow")
+    return {"out": out.view(np.float16), "acc": acc, "codes": codes, "sa": sa}
+
+
+def pack_nibbles(codes: np.ndarray) -> np.ndarray:
+    codes = np.ascontiguousarray(codes, dtype=np.int8)
+    R, K = codes.shape
+    assert K % 2 == 0
+    out = np.empty((R, K // 2), dtype=np.uint8)
+    _load().orc_pack_nibbles(_p(codes), R, K, _p(out))
+    return out
+
+
+def unpack_nibbles(packed: np.ndarray, K: int) -> np.ndarray:
+    packed = np.ascontiguousarray(packed, dtype=np.uint8)
+    R = packed.shape[0]
+    out = np.empty((R, K), dtype=np.int8)
+    _load().orc_unpack_nibbles(_p(packed), R, K, _p(out))
+    return out
+
+
+def residual_stats(x: np.ndarray, dx: np.ndarray, bits: int, eps: float = 1e-6):
+    """(JR_l, SNR_hist_l) of Eqs. 8-11 for one layer's residual state x and update dx [T, d]."""
+    x = np.ascontiguousarray(x, dtype=np.float32)
+    dx = np.ascontiguousarray(dx, dtype=np.float32)
+    T, d = x.shape
+    jr = ctypes.c_double(0)
+    snr = ctypes.c_double(0)
+    if not _load().orc_residual_stats(_p(x), _p(dx), T, d, bits, eps, ctypes.byref(jr),
+                                      ctypes.byref(snr)):
+        raise MemoryError
+    return jr.value, snr.value
