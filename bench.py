@@ -1,0 +1,497 @@
+#!/usr/bin/env python
+"""Benchmark: the LLaMA-2-7B projection stack in decode (32 layers, 4/8-bit activations
+by the layer mask {0, 1, 30, 31}), through the libdptq C ABI on one GB300.
+
+A step is one pass of the whole hot path over one batch of M tokens: for every layer,
+rotate + quantize the qkv input and run the q|k|v GEMM, then o, gate|up and down
+(4 quantizations and 4 GEMMs per layer, 256 kernels per step), replayed as a CUDA
+graph.  The packed weights (3.2 GB) exceed L2, so every step streams them from HBM.
+
+Prints one JSON line (rank 0).  `--impl reference` times the CPU oracle instead on a
+bounded sample of the same workload.  Under torchrun every rank runs an independent
+replica (no collective on the data path); `value` is tokens over all ranks divided by
+the slowest rank's time.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "qlinear TOPS & HBM GB/s (% roofline); 32-layer projection-stack tokens/s"
+UNIT = "tokens/s"
+DEFAULT_M = 32
+
+
+# ------------------------------------------------------------------------------ distributed
+def dist_env():
+    return int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)), int(os.environ.get("LOCAL_RANK", 0))
+
+
+def init_dist(backend):
+    import torch.distributed as dist
+    rank, world, _ = dist_env()
+    if world > 1 and not dist.is_initialized():
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        dist.init_process_group(backend=backend, rank=rank, world_size=world)
+    return rank, world
+
+
+def max_over_ranks(value: float, world: int, device=None) -> float:
+    """Maximum of a per-rank float over all ranks (identity when world == 1)."""
+    if world == 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world: int):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def aggregate_value(tokens_per_rank: int, world: int, t_max_s: float) -> float:
+    """Whole-job throughput: tokens of all ranks over the slowest rank's time."""
+    return tokens_per_rank * world / t_max_s
+
+
+# ------------------------------------------------------------------------------ clocks
+REASONS = {0x1: "gpu_idle", 0x2: "applications_clocks_setting", 0x4: "sw_power_cap", 0x8: "hw_slowdown",
+           0x10: "sync_boost", 0x20: "sw_thermal_slowdown", 0x40: "hw_thermal_slowdown",
+           0x80: "hw_power_brake_slowdown", 0x100: "display_clock_setting"}
+
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons during the timed region."""
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), "--query-gpu=clocks.sm,clocks.max.sm,clocks_event_reasons.active",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except (OSError, ValueError):
+            self.proc = None
+        return self
+
+    def _read(self):
+        for ln in self.proc.stdout:
+            self.lines.append(ln.strip())
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            time.sleep(0.25)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 3:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx = float(parts[1])
+                bits = int(parts[2], 16)
+            except ValueError:
+                continue
+            for b, name in REASONS.items():
+                if bits & b and name != "gpu_idle":
+                    reasons.add(name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": mx, "reasons": ["unsampled"], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ------------------------------------------------------------------------------ workload
+def stack_groups(wl):
+    """(name, K, N, had_block) per activation group of a layer: q|k|v, o, gate|up, down."""
+    out = []
+    for gname, projs in wl.groups():
+        out.append((gname, projs[0].K, sum(p.N for p in projs), projs[0].had_block, [p for p in projs]))
+    return out
+
+
+def build_stack(dp, wl, device):
+    """Pack every layer's weights (seeded, generated on the device) into library handles."""
+    import torch
+    names = [p.name for p in wl.projs]
+    layers = []
+    for layer in range(wl.layers):
+        hs = []
+        for gname, K, N, B, projs in stack_groups(wl):
+            W = torch.cat([_inputs().torch_weights(p.N, p.K, layer, names.index(p.name), device) for p in projs])
+            hs.append(dp.dptq_pack_weights(W.contiguous(), B))
+            del W
+        layers.append(hs)
+    torch.cuda.synchronize()
+    return layers
+
+
+def _inputs():
+    from paper_2606_12487_gb300 import inputs
+    return inputs
+
+
+class Stack:
+    def __init__(self, dp, wl, layers, M, device):
+        import torch
+        self.dp, self.wl, self.layers, self.M = dp, wl, layers, M
+        groups = stack_groups(wl)
+        self.x = [torch.from_numpy(_inputs().activations(wl, M, K, seed=gi)).to(device)
+                  for gi, (_, K, _, _, _) in enumerate(groups)]
+        self.out = [torch.empty((M, N), dtype=torch.float16, device=device) for (_, _, N, _, _) in groups]
+        self.groups = groups
+
+    def run(self, stream, gemm_events=None):
+        """One step (the 32-layer stack).  With gemm_events, record an event pair around
+        every GEMM launch (no graph)."""
+        dp = self.dp
+        for li, hs in enumerate(self.layers):
+            bits = self.wl.bits(li)
+            for gi, h in enumerate(hs):
+                dp.dptq_qlinear_quantize(h, self.x[gi], bits, stream=stream)
+                if gemm_events is not None:
+                    e0, e1 = gemm_events.pop()
+                    e0.record(stream)
+                    dp.dptq_qlinear_gemm(h, self.M, bits, self.out[gi], stream=stream)
+                    e1.record(stream)
+                    gemm_events_done.append((e0, e1, self.gemm_bytes(gi, bits), self.gemm_ops(gi)))
+                else:
+                    dp.dptq_qlinear_gemm(h, self.M, bits, self.out[gi], stream=stream)
+
+    def gemm_bytes(self, gi, bits):
+        """Algorithmic HBM bytes of one GEMM launch: packed int4 weights, weight scales,
+        activation codes at b bits, token scales, fp16 output."""
+        _, K, N, _, _ = self.groups[gi]
+        M = self.M
+        return N * K // 2 + 4 * N + M * K * bits // 8 + 4 * M + 2 * M * N
+
+    def gemm_ops(self, gi):
+        _, K, N, _, _ = self.groups[gi]
+        return 2 * self.M * N * K
+
+    def step_launches(self):
+        return 2 * len(self.groups) * len(self.layers)
+
+    def h2d_bytes(self):
+        return sum(x.numel() * 2 for x in self.x)
+
+    def d2h_bytes(self):
+        return self.out[-1].numel() * 2
+
+
+gemm_events_done = []
+
+
+def time_graph(g, stream, steps, warmup, world, device_index, sample_clocks=True):
+    import torch
+    for _ in range(warmup):
+        g.replay()
+    torch.cuda.synchronize()
+    barrier(world)
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    sampler = ClockSampler(device_index) if sample_clocks else None
+    if sampler:
+        sampler.__enter__()
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(steps):
+            g.replay()
+        e1.record(stream)
+    torch.cuda.synchronize()
+    if sampler:
+        sampler.__exit__(None, None, None)
+    barrier(world)
+    ms = e0.elapsed_time(e1) / steps
+    return ms, (sampler.summary() if sampler else None)
+
+
+def capture(stack, stream):
+    import torch
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        stack.run(stream)
+    torch.cuda.synchronize()
+    return g
+
+
+def measure_gemm_kernels(stack, stream):
+    """Per-launch CUDA-event durations of every GEMM of one eager step (after one warm
+    eager step).  Returns (algorithmic bytes, ops, seconds) summed over the launches."""
+    import torch
+    stack.run(stream)
+    torch.cuda.synchronize()
+    n = len(stack.layers) * len(stack.groups)
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
+    gemm_events_done.clear()
+    stack.run(stream, gemm_events=list(reversed(evs)))
+    torch.cuda.synchronize()
+    tb = to = tt = 0.0
+    per = []
+    for e0, e1, b, o in gemm_events_done:
+        t = e0.elapsed_time(e1) / 1e3
+        tb += b
+        to += o
+        tt += t
+        per.append(t)
+    return tb, to, tt, n
+
+
+def e2e_measure(stack, g, stream, steps, world):
+    """Same metric through the public API with host buffers: per step, H2D copies of
+    the step's inputs from pinned memory, the stack, and a D2H read of the result."""
+    import torch
+    hx = [x.cpu().pin_memory() for x in stack.x]
+    hout = torch.empty(stack.out[-1].shape, dtype=torch.float16).pin_memory()
+    for _ in range(3):
+        with torch.cuda.stream(stream):
+            for h, d in zip(hx, stack.x):
+                d.copy_(h, non_blocking=True)
+        g.replay()
+        with torch.cuda.stream(stream):
+            hout.copy_(stack.out[-1], non_blocking=True)
+    torch.cuda.synchronize()
+    barrier(world)
+    t0 = time.perf_counter()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(steps):
+            for h, d in zip(hx, stack.x):
+                d.copy_(h, non_blocking=True)
+            g.replay()
+            hout.copy_(stack.out[-1], non_blocking=True)
+        e1.record(stream)
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - t0
+    return max(e0.elapsed_time(e1) / 1e3, 0.0) / steps, wall / steps
+
+
+# ------------------------------------------------------------------------------ oracle timing
+def oracle_sample_times(wl, budget_s: float, tokens: int = 1):
+    """Time the oracle's online path (rotate + quantize, int GEMM, epilogue) per layer
+    group at each bit width on `tokens` tokens.  Weight codes are seeded random int4
+    values (packing is offline and not part of the timed path).  Returns
+    {(group, bits): seconds per call} and the number of timed calls."""
+    import numpy as np
+
+    import oracle
+    inputs = _inputs()
+    groups = stack_groups(wl)
+    data = {}
+    for gi, (gname, K, N, B, _) in enumerate(groups):
+        q = inputs.random_codes(N, K, 4, seed=100 + gi)
+        sw = np.full((N,), 0.001, dtype=np.float32)
+        x = inputs.activations(wl, tokens, K, seed=gi)
+        data[gi] = (x, B, q, sw)
+    times = {}
+    calls = 0
+    t_start = time.perf_counter()
+    while True:
+        for gi in data:
+            for bits in (4, 8):
+                x, B, q, sw = data[gi]
+                t0 = time.perf_counter()
+                oracle.qlinear(x, B, bits, q, sw)
+                times.setdefault((gi, bits), []).append(time.perf_counter() - t0)
+                calls += 1
+        if time.perf_counter() - t_start >= budget_s:
+            break
+    return {k: statistics.median(v) for k, v in times.items()}, calls
+
+
+def stack_time_from(wl, times):
+    n_groups = len(stack_groups(wl))
+    return sum(times[(gi, wl.bits(li))] for li in range(wl.layers) for gi in range(n_groups))
+
+
+def cpu_baseline(wl, budget_s=12.0):
+    times, calls = oracle_sample_times(wl, budget_s)
+    t_stack = stack_time_from(wl, times)
+    return {"value": 1.0 / t_stack, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"1 token through each of the 4 projection groups at 4 and 8 bits ({calls} oracle calls, "
+                      f"~{budget_s:.0f} s), weights as random int4 codes; 32-layer stack time summed from the "
+                      "per-group medians with the layer mask"}
+
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if world > 1 and rank != 0:
+        return 0
+    from paper_2606_12487_gb300 import inputs
+    wl = inputs.llama2_7b_decode()
+    # Each step: the oracle on one projection group of one layer for one token, cycling
+    # through the stack; the stack time is assembled from the per-(group, bits) medians.
+    groups = stack_groups(wl)
+    import numpy as np
+
+    import oracle
+    data = []
+    for gi, (gname, K, N, B, _) in enumerate(groups):
+        data.append((inputs.activations(wl, 1, K, seed=gi), B, inputs.random_codes(N, K, 4, seed=100 + gi),
+                     np.full((N,), 0.001, dtype=np.float32)))
+    order = [(li, gi) for li in range(wl.layers) for gi in range(len(groups))]
+    times = {}
+    t_steps = []
+    for i in range(args.warmup + args.steps):
+        li, gi = order[i % len(order)]
+        bits = wl.bits(li)
+        x, B, q, sw = data[gi]
+        t0 = time.perf_counter()
+        oracle.qlinear(x, B, bits, q, sw)
+        dt = time.perf_counter() - t0
+        if i >= args.warmup:
+            times.setdefault((gi, bits), []).append(dt)
+            t_steps.append(dt)
+    for gi in range(len(groups)):
+        for bits in (4, 8):
+            if (gi, bits) not in times:
+                x, B, q, sw = data[gi]
+                t0 = time.perf_counter()
+                oracle.qlinear(x, B, bits, q, sw)
+                times[(gi, bits)] = [time.perf_counter() - t0]
+    med = {k: statistics.median(v) for k, v in times.items()}
+    t_stack = stack_time_from(wl, med)
+    value = 1.0 / t_stack
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * statistics.mean(t_steps),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic",
+        "config": {"workload": "llama2-7b decode projection stack, 32 layers, A8 mask {0,1,30,31}, "
+                               "oracle sample of 1 token per step (one projection group per step)",
+                   "global_batch": 1, "parallelism": "replicas"},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                         "sample": "1 token, one projection group per step cycling through the stack; "
+                                   "stack time from per-(group, bits) medians"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ------------------------------------------------------------------------------ main
+def main(argv=None):
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", default="dptq", choices=["dptq", "reference"])
+    ap.add_argument("--m", type=int, default=DEFAULT_M, help="tokens per step (decode batch)")
+    ap.add_argument("--sweep", default="1,8", help="extra token counts measured for the m_sweep entry")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="run only the first L layers (small cases for profiler captures; 0 = all)")
+    args = ap.parse_args(argv)
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        return run_reference(args)
+
+    import torch
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+    rank, world = init_dist("nccl")
+    from paper_2606_12487_gb300 import dptq, inputs
+    dptq.load()
+    wl = inputs.llama2_7b_decode()
+    if args.layers:
+        wl.layers = min(args.layers, wl.layers)
+    print(f"[bench] rank {rank}/{world}: packing {wl.layers}-layer stack", file=sys.stderr, flush=True)
+    layers = build_stack(dptq, wl, device)
+    max_k = max(K for _, K, _, _, _ in stack_groups(wl))
+    max_m = max([args.m] + [int(v) for v in args.sweep.split(",") if v])
+    dptq.dptq_reserve(max_m, max_k, 0)
+    stream = torch.cuda.Stream(device=device)
+
+    stack = Stack(dptq, wl, layers, args.m, device)
+    g = capture(stack, stream)
+    ms, clocks = time_graph(g, stream, args.steps, args.warmup, world, local)
+    ms_max = max_over_ranks(ms, world, device)
+    value = aggregate_value(args.m, world, ms_max / 1e3)
+
+    tb, to, tt, n_gemm = measure_gemm_kernels(stack, stream)
+    peaks = {}
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            peaks = json.load(f)
+    except OSError:
+        pass
+    hbm_peak = float(peaks.get("hbm_gbs", 6800.0))
+    achieved = tb / tt / 1e9
+    e2e_dev_s, e2e_wall_s = e2e_measure(stack, g, stream, max(10, args.steps // 4), world)
+    e2e_s = max_over_ranks(e2e_dev_s, world, device)
+
+    sweep = {}
+    for m in [int(v) for v in args.sweep.split(",") if v]:
+        st = Stack(dptq, wl, layers, m, device)
+        gm = capture(st, stream)
+        ms_m, _ = time_graph(gm, stream, max(20, args.steps // 2), args.warmup, world, local, sample_clocks=False)
+        ms_m = max_over_ranks(ms_m, world, device)
+        tbm, _, ttm, _ = measure_gemm_kernels(st, stream)
+        sweep[str(m)] = {"tokens_per_s": aggregate_value(m, world, ms_m / 1e3), "ms_per_step": ms_m,
+                         "gemm_gbs": tbm / ttm / 1e9}
+        del gm, st
+    sweep[str(args.m)] = {"tokens_per_s": value, "ms_per_step": ms_max, "gemm_gbs": achieved}
+
+    dptq.dptq_last_device_error()
+    if rank != 0:
+        return 0
+    cpu = None if args.no_cpu_baseline or world > 1 else cpu_baseline(inputs.llama2_7b_decode())
+    weight_bytes = sum(N * K // 2 for _, K, N, _, _ in stack_groups(wl)) * wl.layers
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "int4xint4/int8 (fp8-e4m3 tensor cores, exact int32)", "data": "synthetic",
+        "config": {"workload": f"llama2-7b decode projection stack, {wl.layers} layers, M={args.m} tokens, "
+                               "A8 on layers {0,1,30,31}", "global_batch": args.m * world, "seq_len": 1,
+                   "parallelism": f"replicas x{world}", "l2": "weights 3.24 GB > L2 (streamed every step)",
+                   "weight_bytes_per_step": weight_bytes},
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
+                     "frac": achieved / hbm_peak, "traffic": None, "kernel": "qgemm_kernel",
+                     "peak_source": "MEASURED_PEAKS.json hbm_gbs (copy, burst)",
+                     "launches_per_step": n_gemm},
+        "gemm_tops": to / tt / 1e12,
+        "stack_weight_gbs": weight_bytes / (ms_max / 1e3) / 1e9,
+        "m_sweep": sweep,
+        "e2e": {"value": aggregate_value(args.m, world, e2e_s), "unit": UNIT,
+                "h2d_bytes_per_step": stack.h2d_bytes(), "d2h_bytes_per_step": stack.d2h_bytes(),
+                "wall_ms_per_step": e2e_wall_s * 1e3},
+        "gpu_launches": stack.step_launches() * args.steps,
+        "clocks": clocks,
+        "cpu_baseline": cpu,
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,152 @@
+/*
+ * dptq.h -- C ABI of the GB300 (sm_103a) quantized linear layer of DynamicPTQ
+ * (arxiv 2606.12487): online block-Hadamard rotation of fp16 activations, symmetric
+ * per-token 4/8-bit activation quantization chosen by a per-layer mask, and a GEMM of
+ * packed int4 per-channel weights against the integer codes with exact 32-bit
+ * integer accumulation and a per-token x per-channel scale epilogue to fp16.
+ *
+ * Paper passages the operations follow:
+ *   Section 2, "Low-Bit Quantization of LLMs": Y = X W^T; Q_b(x) = s * round(x / s)
+ *       (Eq. 2); quantization error x - Q_b(x) (Eq. 3).
+ *   Section 2, "Rotation-based Activation Transformation": quantize X R with
+ *       R^T R = I (Eq. 4); fold R into the weight offline, X W^T = (XR)(WR)^T (Eq. 5).
+ *   Section 4.2, "Implementation and Quantization Details": weights per-channel
+ *       symmetric (RTN), activations per-token symmetric, 4 bits by default.
+ *   Section 3.3, Algorithm 1 steps 1-2: weights 4-bit; activations 8-bit on the
+ *       sensitive layers of the mask, 4-bit elsewhere.
+ *
+ * Numerics (readings where the paper is silent):
+ *   R = blockdiag(H_B, ..., H_B, H_r) / sqrt(block) along K, H the Sylvester
+ *   Hadamard matrix in natural order, B = had_block a power of two, r = K mod B a
+ *   power of two (or 0).  Scales s = max|row| / (2^(b-1) - 1) in fp32 (IEEE
+ *   division); codes round half to even, clamped to [-2^(b-1), 2^(b-1) - 1];
+ *   an all-zero row has s = 0 and all codes 0.  Output
+ *   out[m][n] = fp16_rne( fp32( fp32(acc[m][n]) * s_a[m] ) * s_w[n] ).
+ *
+ * Conventions for every call:
+ *   - Pointers passed to the online calls are DEVICE pointers owned by the caller;
+ *     the library never frees them.  fp16 buffers are raw IEEE binary16 (uint16_t).
+ *     Activation and output matrices are row-major and dense; x and codes rows must
+ *     start 16-byte aligned (true for dense rows when K % 32 == 0 and the base
+ *     pointer is 16-byte aligned).
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
+ *     Online calls are asynchronous and stream-ordered; they do not synchronize the
+ *     host.  Calls that share one handle, or the library scratch of one device,
+ *     must not run concurrently on different streams.
+ *   - Shape rules: 1 <= K, K % 32 == 0, N % 16 == 0, K splits into blocks of
+ *     had_block plus a power-of-two tail, bits in {4, 8}.  Violations return
+ *     DPTQ_ERR_INVALID_ARG (bits, null pointers, negative sizes) or
+ *     DPTQ_ERR_UNSUPPORTED (shape).  M == 0 is a no-op.
+ *   - No exception crosses this boundary.  CUDA errors map to DPTQ_ERR_CUDA; the
+ *     message of the last failure on the calling thread is dptq_last_error_message().
+ *   - Device-side waits are bounded: a pipeline wait that exceeds about one second
+ *     makes the kernel record an error word and return; dptq_last_device_error()
+ *     reports it as DPTQ_ERR_TIMEOUT.
+ */
+#ifndef DPTQ_H_
+#define DPTQ_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  DPTQ_OK = 0,
+  DPTQ_ERR_INVALID_ARG = 1,
+  DPTQ_ERR_UNSUPPORTED = 2,
+  DPTQ_ERR_CUDA = 3,
+  DPTQ_ERR_OOM = 4,
+  DPTQ_ERR_TIMEOUT = 5
+} dptq_status;
+
+/* Opaque handle of one quantized linear layer.  It owns the packed weights, the
+ * per-channel scales and the shape; it is created by dptq_pack_weights and released
+ * by dptq_destroy. */
+typedef struct dptq_linear* dptq_handle;
+
+/* Offline weight packing (Section 2 Eq. 5; Section 4.2 RTN per-channel symmetric).
+ * W_fp16: [N][K] row-major binary16 weights, on the device if w_on_device != 0,
+ *   else in host memory.  Read only; not retained.
+ * Computes W' = W R, s_w[n] = max_k |W'[n][k]| / 7, q = clamp(rint(W'/s_w), -8, 7)
+ * on the GPU and keeps q (4 bits per weight, in a tiled device layout) and s_w in
+ * device memory owned by the handle.  Synchronous (returns after packing).
+ * Errors: INVALID_ARG for null pointers or sizes <= 0, UNSUPPORTED for shapes, OOM
+ * when device memory runs out, CUDA for other CUDA failures. */
+dptq_status dptq_pack_weights(const void* W_fp16, int N, int K, int had_block, int w_on_device,
+                              dptq_handle* out);
+
+/* Online rotation + quantization of activations (Section 2 Eq. 4 then Eq. 2).
+ * x_fp16: device [M][K] binary16.  bits: 4 or 8 (the mask entry of the layer).
+ * codes (device, written): bits == 4: uint8 [M][K/2], byte j of a row holds code 2j in
+ *   bits 0-3 and code 2j+1 in bits 4-7, each 4-bit two's complement;
+ *   bits == 8: int8 [M][K].
+ * scales (device, written): float [M], s_a per token.
+ * One fused kernel: 128-bit loads, Walsh-Hadamard butterflies in fp32, row absmax,
+ * rounding, packing. */
+dptq_status dptq_rotate_quant_act(const void* x_fp16, int M, int K, int had_block, int bits,
+                                  void* codes, float* scales, void* stream);
+
+/* Test hook: the rotated activations y = x R as fp32 [M][K] (device), the value the
+ * quantizer of dptq_rotate_quant_act sees. */
+dptq_status dptq_rotate_act(const void* x_fp16, int M, int K, int had_block, float* y_f32,
+                            void* stream);
+
+/* The quantized linear layer: out = fp16( Q(x R) (W R)^T scaled ), i.e. rotate and
+ * quantize x with `bits` (4 or 8, the layer's mask entry), multiply by the packed
+ * int4 weights of `h` with exact int32 accumulation, apply s_a[m] * s_w[n].
+ * x_fp16: device [M][K]; out_fp16: device [M][N] (written).  Asynchronous.
+ * Uses the library's per-device scratch (grown on demand; call dptq_reserve before
+ * capturing into a CUDA graph so that no allocation happens during capture). */
+dptq_status dptq_qlinear(dptq_handle h, const void* x_fp16, int M, int bits, void* out_fp16,
+                         void* stream);
+
+/* The two halves of dptq_qlinear, for callers that feed one quantized activation
+ * matrix to several layers with the same K and had_block (for example q, k and v):
+ * dptq_qlinear_quantize rotates and quantizes x into the device's scratch (the same
+ * kernel as dptq_rotate_quant_act, writing the GEMM's operand layout), and
+ * dptq_qlinear_gemm multiplies those codes by the weights of `h`.  The codes stay in
+ * the scratch until the next quantize call on the device; a gemm call must use the
+ * M and bits of the preceding quantize call and a handle with its K and had_block. */
+dptq_status dptq_qlinear_quantize(dptq_handle h, const void* x_fp16, int M, int bits, void* stream);
+dptq_status dptq_qlinear_gemm(dptq_handle h, int M, int bits, void* out_fp16, void* stream);
+
+/* GEMM + epilogue on caller-provided codes (the format dptq_rotate_quant_act writes)
+ * and per-token scales.  acc_i32: optional device int32 [M][N] that receives the
+ * exact integer accumulators (test hook); NULL to skip. */
+dptq_status dptq_qgemm_codes(dptq_handle h, const void* codes, const float* scales, int M, int bits,
+                             void* out_fp16, int32_t* acc_i32, void* stream);
+
+/* Pre-size the per-device scratch for calls with up to max_M tokens and up to max_K
+ * inputs / max_N outputs, so that later calls allocate nothing.  Synchronous. */
+dptq_status dptq_reserve(int max_M, int max_K, int max_N);
+
+/* Copy the packed weights out in the public layout: wq_host uint8 [N][K/2] (same
+ * nibble format as 4-bit activation codes) and sw_host float [N].  Either may be
+ * NULL.  Synchronous (test access). */
+dptq_status dptq_get_packed(dptq_handle h, void* wq_host, float* sw_host);
+
+/* Shape of a handle (any pointer may be NULL). */
+dptq_status dptq_get_shape(dptq_handle h, int* N, int* K, int* had_block);
+
+/* Synchronize the device and report (and clear) the device error word set by a
+ * bounded wait that gave up: DPTQ_OK or DPTQ_ERR_TIMEOUT.  `h` may be NULL. */
+dptq_status dptq_last_device_error(dptq_handle h);
+
+/* Release a handle and its device memory.  NULL is ignored.  Must not be called
+ * while work using the handle is still running. */
+void dptq_destroy(dptq_handle h);
+
+/* Static description of a status code. */
+const char* dptq_status_str(dptq_status s);
+
+/* Message of the last failing call on this thread ("" if none). */
+const char* dptq_last_error_message(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DPTQ_H_ */

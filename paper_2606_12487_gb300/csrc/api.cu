@@ -1,0 +1,458 @@
+// api.cu -- the C ABI of include/dptq.h: argument checks, the layer handle, the
+// per-device scratch, and the launch sequence of each call.  No compute happens here;
+// every step of the path runs in the kernels of rotate_quant.cu and qgemm.cu.
+#include <cmath>
+#include <cstdint>
+#include <cstdio>
+#include <cstring>
+#include <map>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include <cuda_runtime.h>
+
+#include "../../include/dptq.h"
+#include "dptq_internal.h"
+
+using namespace dptq;
+
+struct dptq_linear {
+  int device;
+  int N, K, K_pad, KB, N_pad;
+  int had_block;
+  uint8_t* wt;  // [N_pad/128][KB][128][64] sign-magnitude nibbles
+  float* sw;    // [N_pad]
+};
+
+namespace {
+
+thread_local std::string g_msg;
+
+dptq_status fail(dptq_status st, const std::string& m) {
+  g_msg = m;
+  return st;
+}
+dptq_status cuda_fail(cudaError_t e, const char* where) {
+  g_msg = std::string(where) + ": " + cudaGetErrorString(e);
+  return e == cudaErrorMemoryAllocation ? DPTQ_ERR_OOM : DPTQ_ERR_CUDA;
+}
+#define DPTQ_CUDA(call, where)                      \
+  do {                                              \
+    cudaError_t e_ = (call);                        \
+    if (e_ != cudaSuccess) return cuda_fail(e_, where); \
+  } while (0)
+
+bool is_pow2(int v) { return v > 0 && (v & (v - 1)) == 0; }
+
+// Block layout of R along K: nfull blocks of B then a power-of-two tail (or none).
+bool hadamard_layout(int K, int B, int& nfull, int& tail, int& log2B) {
+  if (!is_pow2(B) || K <= 0) return false;
+  nfull = K / B;
+  tail = K % B;
+  if (tail != 0 && !is_pow2(tail)) return false;
+  log2B = 0;
+  while ((1 << log2B) < B) ++log2B;
+  return true;
+}
+
+// Elements per rotation pass: whole blocks, at least 4096 elements when K allows.
+int rq_chunk(int K, int B) {
+  int c = B;
+  while (c < 4096 && c < K) c += B;
+  return c < K ? c : K;
+}
+
+dptq_status check_shape(int K, int B, int& nfull, int& tail, int& log2B) {
+  if (K % 32 != 0) return fail(DPTQ_ERR_UNSUPPORTED, "K must be a multiple of 32");
+  if (!hadamard_layout(K, B, nfull, tail, log2B))
+    return fail(DPTQ_ERR_UNSUPPORTED, "K must split into blocks of had_block (a power of two) plus a power-of-two tail");
+  if (rotate_quant_smem(K, rq_chunk(K, B)) > kSmemPerBlock)
+    return fail(DPTQ_ERR_UNSUPPORTED, "K and had_block exceed the shared memory of one CTA");
+  return DPTQ_OK;
+}
+
+RQArgs make_rq(const void* x, int rows_in, int rows_out, int K, int KB, int B, int nfull, int tail, int log2B,
+               int bits, float* scales, void* out) {
+  RQArgs a{};
+  a.x = static_cast<const __half*>(x);
+  a.rows_in = rows_in;
+  a.rows_out = rows_out;
+  a.K = K;
+  a.KB = KB;
+  a.B = B;
+  a.log2B = log2B;
+  a.nfull = nfull;
+  a.tail = tail;
+  a.log2T = 0;
+  while (tail && (1 << a.log2T) < tail) ++a.log2T;
+  a.chunk = rq_chunk(K, B);
+  const double r2 = 1.0 / std::sqrt(2.0);
+  a.c_hi = (float)r2;
+  a.c_lo = (float)(r2 - (double)a.c_hi);
+  a.bits = bits;
+  a.scales = scales;
+  a.out = out;
+  return a;
+}
+
+// Per-device scratch shared by the online calls: E4M3 activation planes, per-token
+// scales, split-tile partial sums and their counters, and the device error word.
+struct Scratch {
+  uint8_t* act = nullptr;
+  size_t act_bytes = 0;
+  float* sa = nullptr;
+  size_t sa_count = 0;
+  int32_t* ws = nullptr;
+  uint32_t* counters = nullptr;
+  int* err = nullptr;
+  int num_sms = 0;
+};
+std::mutex g_mu;
+std::map<int, Scratch> g_scratch;
+
+bool capturing(cudaStream_t s) {
+  cudaStreamCaptureStatus st = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(s, &st) != cudaSuccess) return false;
+  return st != cudaStreamCaptureStatusNone;
+}
+
+constexpr int kMaxNT = 256;
+
+// Make sure the device's scratch holds `act_bytes` of activation planes and `sa_count`
+// scales.  Growth allocates, so it is refused while `s` is being captured.
+dptq_status ensure_scratch(int dev, size_t act_bytes, size_t sa_count, cudaStream_t s, Scratch** out) {
+  std::lock_guard<std::mutex> lk(g_mu);
+  Scratch& sc = g_scratch[dev];
+  const bool grow_act = act_bytes > sc.act_bytes;
+  const bool grow_sa = sa_count > sc.sa_count;
+  const bool first = sc.err == nullptr;
+  if ((grow_act || grow_sa || first) && capturing(s))
+    return fail(DPTQ_ERR_UNSUPPORTED, "scratch must grow during stream capture: call dptq_reserve first");
+  if (first) {
+    DPTQ_CUDA(cudaDeviceGetAttribute(&sc.num_sms, cudaDevAttrMultiProcessorCount, dev), "cudaDeviceGetAttribute");
+    const size_t ws_bytes = (size_t)sc.num_sms * kMaxNT * 128 * sizeof(int32_t);
+    DPTQ_CUDA(cudaMalloc(&sc.ws, ws_bytes), "cudaMalloc(ws)");
+    DPTQ_CUDA(cudaMalloc(&sc.counters, sizeof(uint32_t) * sc.num_sms), "cudaMalloc(counters)");
+    DPTQ_CUDA(cudaMalloc(&sc.err, sizeof(int)), "cudaMalloc(err)");
+    DPTQ_CUDA(cudaMemset(sc.ws, 0, ws_bytes), "cudaMemset(ws)");
+    DPTQ_CUDA(cudaMemset(sc.counters, 0, sizeof(uint32_t) * sc.num_sms), "cudaMemset(counters)");
+    DPTQ_CUDA(cudaMemset(sc.err, 0, sizeof(int)), "cudaMemset(err)");
+  }
+  if (grow_act || grow_sa) DPTQ_CUDA(cudaDeviceSynchronize(), "cudaDeviceSynchronize");
+  if (grow_act) {
+    if (sc.act) cudaFree(sc.act);
+    sc.act = nullptr;
+    sc.act_bytes = 0;
+    DPTQ_CUDA(cudaMalloc(&sc.act, act_bytes), "cudaMalloc(act)");
+    sc.act_bytes = act_bytes;
+  }
+  if (grow_sa) {
+    if (sc.sa) cudaFree(sc.sa);
+    sc.sa = nullptr;
+    sc.sa_count = 0;
+    DPTQ_CUDA(cudaMalloc(&sc.sa, sizeof(float) * sa_count), "cudaMalloc(sa)");
+    sc.sa_count = sa_count;
+  }
+  *out = &sc;
+  return DPTQ_OK;
+}
+
+dptq_status current_device(int* dev) {
+  DPTQ_CUDA(cudaGetDevice(dev), "cudaGetDevice");
+  return DPTQ_OK;
+}
+
+dptq_status check_handle(dptq_handle h, int* dev) {
+  if (!h) return fail(DPTQ_ERR_INVALID_ARG, "null handle");
+  dptq_status st = current_device(dev);
+  if (st != DPTQ_OK) return st;
+  if (*dev != h->device) return fail(DPTQ_ERR_INVALID_ARG, "handle belongs to another device than the current one");
+  return DPTQ_OK;
+}
+
+// GEMM + epilogue from the E4M3 planes already in scratch.
+dptq_status run_gemm(dptq_handle h, const GemmPlan& plan0, const uint8_t* act, const float* sa, void* out,
+                     int32_t* acc, Scratch* sc, cudaStream_t s) {
+  GemmPlan plan = plan0;
+  GemmArgs& g = plan.args;
+  g.wt = h->wt;
+  g.act = act;
+  g.sa = sa;
+  g.sw = h->sw;
+  g.out = static_cast<__half*>(out);
+  g.acc_out = acc;
+  g.ws = sc->ws;
+  g.counters = sc->counters;
+  g.err = sc->err;
+  DPTQ_CUDA(launch_gemm(plan, s, true), "qgemm launch");
+  return DPTQ_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* dptq_status_str(dptq_status s) {
+  switch (s) {
+    case DPTQ_OK: return "ok";
+    case DPTQ_ERR_INVALID_ARG: return "invalid argument";
+    case DPTQ_ERR_UNSUPPORTED: return "unsupported shape";
+    case DPTQ_ERR_CUDA: return "CUDA error";
+    case DPTQ_ERR_OOM: return "out of device memory";
+    case DPTQ_ERR_TIMEOUT: return "device wait timed out";
+  }
+  return "unknown status";
+}
+
+const char* dptq_last_error_message(void) { return g_msg.c_str(); }
+
+dptq_status dptq_pack_weights(const void* W_fp16, int N, int K, int had_block, int w_on_device, dptq_handle* out) {
+  if (!W_fp16 || !out) return fail(DPTQ_ERR_INVALID_ARG, "null pointer");
+  *out = nullptr;
+  if (N <= 0 || K <= 0 || had_block <= 0) return fail(DPTQ_ERR_INVALID_ARG, "sizes must be positive");
+  if (N % 16 != 0) return fail(DPTQ_ERR_UNSUPPORTED, "N must be a multiple of 16");
+  int nfull, tail, log2B;
+  dptq_status st = check_shape(K, had_block, nfull, tail, log2B);
+  if (st != DPTQ_OK) return st;
+  int dev;
+  if ((st = current_device(&dev)) != DPTQ_OK) return st;
+
+  dptq_linear* h = new dptq_linear{};
+  h->device = dev;
+  h->N = N;
+  h->K = K;
+  h->K_pad = round_up(K, kKBlock);
+  h->KB = h->K_pad / kKBlock;
+  h->N_pad = round_up(N, 128);
+  h->had_block = had_block;
+  const size_t wt_bytes = (size_t)(h->N_pad / 128) * h->KB * kWTileBytes;
+  void* tmp = nullptr;
+  cudaError_t e = cudaMalloc(&h->wt, wt_bytes);
+  if (e == cudaSuccess) e = cudaMalloc(&h->sw, sizeof(float) * h->N_pad);
+  const void* src = W_fp16;
+  if (e == cudaSuccess && !w_on_device) {
+    e = cudaMalloc(&tmp, (size_t)N * K * 2);
+    if (e == cudaSuccess) e = cudaMemcpy(tmp, W_fp16, (size_t)N * K * 2, cudaMemcpyHostToDevice);
+    src = tmp;
+  }
+  if (e == cudaSuccess) {
+    RQArgs a = make_rq(src, N, h->N_pad, K, h->KB, had_block, nfull, tail, log2B, 4, h->sw, h->wt);
+    e = launch_rotate_quant(kRQWeights, a, 0, false);
+  }
+  if (e == cudaSuccess) e = cudaDeviceSynchronize();
+  if (tmp) cudaFree(tmp);
+  if (e != cudaSuccess) {
+    dptq_destroy(h);
+    return cuda_fail(e, "dptq_pack_weights");
+  }
+  *out = h;
+  return DPTQ_OK;
+}
+
+dptq_status dptq_rotate_quant_act(const void* x_fp16, int M, int K, int had_block, int bits, void* codes,
+                                  float* scales, void* stream) {
+  if (bits != 4 && bits != 8) return fail(DPTQ_ERR_INVALID_ARG, "bits must be 4 or 8");
+  if (M < 0 || K <= 0 || had_block <= 0) return fail(DPTQ_ERR_INVALID_ARG, "bad sizes");
+  if (M == 0) return DPTQ_OK;
+  if (!x_fp16 || !codes || !scales) return fail(DPTQ_ERR_INVALID_ARG, "null pointer");
+  int nfull, tail, log2B;
+  dptq_status st = check_shape(K, had_block, nfull, tail, log2B);
+  if (st != DPTQ_OK) return st;
+  RQArgs a = make_rq(x_fp16, M, M, K, round_up(K, kKBlock) / kKBlock, had_block, nfull, tail, log2B, bits, scales,
+                     codes);
+  DPTQ_CUDA(launch_rotate_quant(kRQPublic, a, static_cast<cudaStream_t>(stream), true), "rotate_quant launch");
+  return DPTQ_OK;
+}
+
+dptq_status dptq_rotate_act(const void* x_fp16, int M, int K, int had_block, float* y_f32, void* stream) {
+  if (M < 0 || K <= 0 || had_block <= 0) return fail(DPTQ_ERR_INVALID_ARG, "bad sizes");
+  if (M == 0) return DPTQ_OK;
+  if (!x_fp16 || !y_f32) return fail(DPTQ_ERR_INVALID_ARG, "null pointer");
+  int nfull, tail, log2B;
+  dptq_status st = check_shape(K, had_block, nfull, tail, log2B);
+  if (st != DPTQ_OK) return st;
+  RQArgs a = make_rq(x_fp16, M, M, K, round_up(K, kKBlock) / kKBlock, had_block, nfull, tail, log2B, 4, nullptr,
+                     y_f32);
+  DPTQ_CUDA(launch_rotate_quant(kRQY, a, static_cast<cudaStream_t>(stream), true), "rotate launch");
+  return DPTQ_OK;
+}
+
+}  // extern "C"
+
+namespace {
+
+// Shape checks and scratch sizing shared by the qlinear entry points.
+dptq_status prepare_qlinear(dptq_handle h, int M, int bits, cudaStream_t s, int* dev, GemmPlan* plan,
+                            Scratch** sc) {
+  if (bits != 4 && bits != 8) return fail(DPTQ_ERR_INVALID_ARG, "bits must be 4 or 8");
+  if (M < 0) return fail(DPTQ_ERR_INVALID_ARG, "M must be >= 0");
+  dptq_status st = check_handle(h, dev);
+  if (st != DPTQ_OK) return st;
+  if (M == 0) return DPTQ_OK;
+  if ((st = ensure_scratch(*dev, 0, 0, s, sc)) != DPTQ_OK) return st;
+  if (!plan_gemm(M, h->N, h->K_pad, bits, (*sc)->num_sms, *plan)) return fail(DPTQ_ERR_UNSUPPORTED, "no GEMM plan");
+  const int planes = bits == 8 ? 2 : 1;
+  return ensure_scratch(*dev, (size_t)planes * h->K_pad * plan->M_pad, plan->M_pad, s, sc);
+}
+
+dptq_status quantize_into_scratch(dptq_handle h, const void* x_fp16, int M, int bits, const GemmPlan& plan,
+                                  Scratch* sc, cudaStream_t s) {
+  int nfull, tail, log2B;
+  dptq_status st = check_shape(h->K, h->had_block, nfull, tail, log2B);
+  if (st != DPTQ_OK) return st;
+  RQArgs a = make_rq(x_fp16, M, plan.M_pad, h->K, h->KB, h->had_block, nfull, tail, log2B, bits, sc->sa, sc->act);
+  DPTQ_CUDA(launch_rotate_quant(kRQAct, a, s, true), "rotate_quant launch");
+  return DPTQ_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+dptq_status dptq_qlinear(dptq_handle h, const void* x_fp16, int M, int bits, void* out_fp16, void* stream) {
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  int dev;
+  GemmPlan plan;
+  Scratch* sc = nullptr;
+  dptq_status st = prepare_qlinear(h, M, bits, s, &dev, &plan, &sc);
+  if (st != DPTQ_OK || M == 0) return st;
+  if (!x_fp16 || !out_fp16) return fail(DPTQ_ERR_INVALID_ARG, "null pointer");
+  if ((st = quantize_into_scratch(h, x_fp16, M, bits, plan, sc, s)) != DPTQ_OK) return st;
+  return run_gemm(h, plan, sc->act, sc->sa, out_fp16, nullptr, sc, s);
+}
+
+dptq_status dptq_qlinear_quantize(dptq_handle h, const void* x_fp16, int M, int bits, void* stream) {
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  int dev;
+  GemmPlan plan;
+  Scratch* sc = nullptr;
+  dptq_status st = prepare_qlinear(h, M, bits, s, &dev, &plan, &sc);
+  if (st != DPTQ_OK || M == 0) return st;
+  if (!x_fp16) return fail(DPTQ_ERR_INVALID_ARG, "null pointer");
+  return quantize_into_scratch(h, x_fp16, M, bits, plan, sc, s);
+}
+
+dptq_status dptq_qlinear_gemm(dptq_handle h, int M, int bits, void* out_fp16, void* stream) {
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  int dev;
+  GemmPlan plan;
+  Scratch* sc = nullptr;
+  dptq_status st = prepare_qlinear(h, M, bits, s, &dev, &plan, &sc);
+  if (st != DPTQ_OK || M == 0) return st;
+  if (!out_fp16) return fail(DPTQ_ERR_INVALID_ARG, "null pointer");
+  return run_gemm(h, plan, sc->act, sc->sa, out_fp16, nullptr, sc, s);
+}
+
+dptq_status dptq_qgemm_codes(dptq_handle h, const void* codes, const float* scales, int M, int bits, void* out_fp16,
+                             int32_t* acc_i32, void* stream) {
+  if (bits != 4 && bits != 8) return fail(DPTQ_ERR_INVALID_ARG, "bits must be 4 or 8");
+  if (M < 0) return fail(DPTQ_ERR_INVALID_ARG, "M must be >= 0");
+  int dev;
+  dptq_status st = check_handle(h, &dev);
+  if (st != DPTQ_OK) return st;
+  if (M == 0) return DPTQ_OK;
+  if (!codes || !scales || !out_fp16) return fail(DPTQ_ERR_INVALID_ARG, "null pointer");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  Scratch* sc = nullptr;
+  if ((st = ensure_scratch(dev, 0, 0, s, &sc)) != DPTQ_OK) return st;
+  GemmPlan plan;
+  if (!plan_gemm(M, h->N, h->K_pad, bits, sc->num_sms, plan)) return fail(DPTQ_ERR_UNSUPPORTED, "no GEMM plan");
+  const int planes = bits == 8 ? 2 : 1;
+  if ((st = ensure_scratch(dev, (size_t)planes * h->K_pad * plan.M_pad, 0, s, &sc)) != DPTQ_OK) return st;
+  CodesArgs c{};
+  c.codes = static_cast<const uint8_t*>(codes);
+  c.M = M;
+  c.M_pad = plan.M_pad;
+  c.K = h->K;
+  c.KB = h->KB;
+  c.bits = bits;
+  c.act = sc->act;
+  DPTQ_CUDA(launch_codes_to_act(c, s), "codes_to_act launch");
+  return run_gemm(h, plan, sc->act, scales, out_fp16, acc_i32, sc, s);
+}
+
+dptq_status dptq_reserve(int max_M, int max_K, int max_N) {
+  if (max_M < 0 || max_K < 0 || max_N < 0) return fail(DPTQ_ERR_INVALID_ARG, "sizes must be >= 0");
+  int dev;
+  dptq_status st = current_device(&dev);
+  if (st != DPTQ_OK) return st;
+  (void)max_N;
+  const size_t M_pad = (size_t)round_up(max_M > 0 ? max_M : 1, kMaxNT);
+  const size_t K_pad = (size_t)round_up(max_K > 0 ? max_K : kKBlock, kKBlock);
+  Scratch* sc = nullptr;
+  st = ensure_scratch(dev, 2 * K_pad * M_pad, M_pad, 0, &sc);
+  if (st != DPTQ_OK) return st;
+  DPTQ_CUDA(cudaDeviceSynchronize(), "cudaDeviceSynchronize");
+  return DPTQ_OK;
+}
+
+dptq_status dptq_get_packed(dptq_handle h, void* wq_host, float* sw_host) {
+  int dev;
+  dptq_status st = check_handle(h, &dev);
+  if (st != DPTQ_OK) return st;
+  if (sw_host) DPTQ_CUDA(cudaMemcpy(sw_host, h->sw, sizeof(float) * h->N, cudaMemcpyDeviceToHost), "cudaMemcpy(sw)");
+  if (!wq_host) return DPTQ_OK;
+  const size_t wt_bytes = (size_t)(h->N_pad / 128) * h->KB * kWTileBytes;
+  std::vector<uint8_t> t(wt_bytes);
+  DPTQ_CUDA(cudaMemcpy(t.data(), h->wt, wt_bytes, cudaMemcpyDeviceToHost), "cudaMemcpy(wt)");
+  uint8_t* dst = static_cast<uint8_t*>(wq_host);
+  for (int n = 0; n < h->N; ++n) {
+    for (int k = 0; k < h->K; k += 2) {
+      int code[2];
+      for (int d = 0; d < 2; ++d) {
+        const int kk = k + d;
+        const int e = kk & 15;  // position in the 16-weight chunk
+        const size_t chunk = (((size_t)(n >> 7) * h->KB + (kk >> 7)) * kWTileBytes) + (n & 127) * 64 +
+                             ((kk & 127) >> 4) * 8;
+        const int word = e >> 3, i = e & 3, high = (e & 7) >= 4;
+        const uint8_t byte = t[chunk + word * 4 + i];
+        const int nib = high ? (byte >> 4) & 0xF : byte & 0xF;
+        const int mag = nib & 7;
+        code[d] = (nib & 8) ? -mag : mag;
+      }
+      dst[(size_t)n * (h->K / 2) + k / 2] = (uint8_t)((code[0] & 0xF) | ((code[1] & 0xF) << 4));
+    }
+  }
+  return DPTQ_OK;
+}
+
+dptq_status dptq_get_shape(dptq_handle h, int* N, int* K, int* had_block) {
+  if (!h) return fail(DPTQ_ERR_INVALID_ARG, "null handle");
+  if (N) *N = h->N;
+  if (K) *K = h->K;
+  if (had_block) *had_block = h->had_block;
+  return DPTQ_OK;
+}
+
+dptq_status dptq_last_device_error(dptq_handle h) {
+  (void)h;
+  int dev;
+  dptq_status st = current_device(&dev);
+  if (st != DPTQ_OK) return st;
+  DPTQ_CUDA(cudaDeviceSynchronize(), "cudaDeviceSynchronize");
+  std::lock_guard<std::mutex> lk(g_mu);
+  auto it = g_scratch.find(dev);
+  if (it == g_scratch.end() || it->second.err == nullptr) return DPTQ_OK;
+  Scratch& sc = it->second;
+  int word = 0;
+  DPTQ_CUDA(cudaMemcpy(&word, sc.err, sizeof(int), cudaMemcpyDeviceToHost), "cudaMemcpy(err)");
+  if (word == 0) return DPTQ_OK;
+  // A wait gave up: clear the word and the split-tile scratch the aborted kernel may
+  // have left non-zero.
+  DPTQ_CUDA(cudaMemset(sc.err, 0, sizeof(int)), "cudaMemset(err)");
+  DPTQ_CUDA(cudaMemset(sc.ws, 0, (size_t)sc.num_sms * kMaxNT * 128 * sizeof(int32_t)), "cudaMemset(ws)");
+  DPTQ_CUDA(cudaMemset(sc.counters, 0, sizeof(uint32_t) * sc.num_sms), "cudaMemset(counters)");
+  char buf[64];
+  snprintf(buf, sizeof(buf), "device wait timed out (code 0x%x)", word);
+  return fail(DPTQ_ERR_TIMEOUT, buf);
+}
+
+void dptq_destroy(dptq_handle h) {
+  if (!h) return;
+  if (h->wt) cudaFree(h->wt);
+  if (h->sw) cudaFree(h->sw);
+  delete h;
+}
+
+}  // extern "C"

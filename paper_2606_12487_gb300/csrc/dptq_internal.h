@@ -1,0 +1,95 @@
+// dptq_internal.h -- host-side declarations shared by the CUDA translation units of
+// libdptq (kernel argument blocks and launchers).  Not part of the public ABI.
+#pragma once
+#include <cstdint>
+#include <cuda_runtime.h>
+#include <cuda_fp16.h>
+
+namespace dptq {
+
+// K is processed in blocks of 128 elements: one 128-byte row of the MMA's swizzled
+// FP8 operand tile.
+constexpr int kKBlock = 128;
+// One (128 output channels) x (128 k) tile of packed 4-bit weights.
+constexpr int kWTileBytes = 128 * 64;
+
+inline int ceil_div(long long a, long long b) { return (int)((a + b - 1) / b); }
+inline int round_up(int a, int b) { return ceil_div(a, b) * b; }
+
+// ------------------------------------------------------------------ rotate + quantize
+enum RQMode : int {
+  kRQPublic = 0,   // codes in the public format (A4 packed nibbles / A8 int8) + scales
+  kRQAct = 1,      // codes as E4M3 planes in the GEMM's swizzled tile layout + scales
+  kRQY = 2,        // rotated fp32 activations (test hook)
+  kRQWeights = 3,  // packed sign-magnitude int4 weight tiles + per-channel scales
+};
+
+struct RQArgs {
+  const __half* x;   // [rows_in][K] binary16, row-major
+  int rows_in;       // rows that carry data (M tokens or N channels)
+  int rows_out;      // rows written (padded; rows >= rows_in are zero)
+  int K;             // logical K
+  int KB;            // K_pad / 128
+  int B;             // Hadamard block size (power of two)
+  int log2B;
+  int nfull;         // number of whole blocks of size B
+  int tail;          // tail block size (power of two) or 0
+  int log2T;         // log2(tail) (0 when there is no tail)
+  int chunk;         // elements rotated per shared-memory pass (a multiple of B)
+  float c_hi, c_lo;  // 1/sqrt(2) as an fp32 pair (c_hi + c_lo to ~2^-48)
+  int bits;          // 4 or 8
+  float* scales;     // [rows_out] (rows >= rows_in get 0); may be null in kRQY
+  void* out;         // mode-dependent destination
+};
+
+cudaError_t launch_rotate_quant(RQMode mode, const RQArgs& a, cudaStream_t s, bool pdl);
+size_t rotate_quant_smem(int K, int chunk);
+// Shared-memory budget of one CTA (227 KB opt-in).
+constexpr size_t kSmemPerBlock = 232448;
+
+// Public codes (A4 packed two's complement / A8 int8) -> E4M3 GEMM planes.
+struct CodesArgs {
+  const uint8_t* codes;
+  int M, M_pad, K, KB, bits;
+  uint8_t* act;
+};
+cudaError_t launch_codes_to_act(const CodesArgs& a, cudaStream_t s);
+
+// ------------------------------------------------------------------ GEMM
+struct GemmArgs {
+  const uint8_t* wt;   // [NTw][KB][128][64] packed sign-magnitude nibbles
+  const uint8_t* act;  // [planes][KB][M_pad][128] E4M3, rows pre-swizzled
+  const float* sa;     // [>= M] per-token scales
+  const float* sw;     // [>= N] per-channel scales
+  __half* out;         // [M][N]
+  int32_t* acc_out;    // optional [M][N]
+  int32_t* ws;         // split-tile partial sums: [grid][NT * 128]
+  uint32_t* counters;  // [grid] arrival counters (zero between launches)
+  int* err;            // device error word
+  int M, N, M_pad, KB, planes;
+  int n_wtiles;        // N_pad / 128
+  int m_tiles;         // M_pad / NT
+  int seg_blocks;      // k-blocks per exact fp32 accumulation segment
+  int segs;            // accumulator segments per tile
+  int nbuf;            // TMEM accumulator buffers (1 or 2)
+  int stages;          // shared-memory pipeline depth
+  int dp_tiles;        // tiles processed whole, round-robin, before the stream-K part
+  long long sk_iters;  // stream-K iterations (tiles after dp_tiles, times KB)
+  uint32_t tmem_cols;
+};
+
+struct GemmPlan {
+  int nt;          // token tile (MMA N): 16, 32, 64, 128 or 256
+  int M_pad;
+  int grid;
+  int smem_bytes;
+  GemmArgs args;
+};
+
+// Fills everything in `plan.args` that depends only on shapes; the caller sets the
+// pointers.  Returns false if the shape cannot be run.
+bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan);
+cudaError_t launch_gemm(const GemmPlan& plan, cudaStream_t s, bool pdl);
+int gemm_pick_nt(int M, int bits, int KB);
+
+}  // namespace dptq

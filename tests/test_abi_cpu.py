@@ -1,0 +1,80 @@
+"""C-ABI library checks that need no GPU: it builds for sm_103a, loads, exports every
+function include/dptq.h declares, and rejects bad arguments before touching CUDA."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2606_12487_gb300 import dptq
+    return dptq.load()
+
+
+def declared_functions():
+    names = []
+    for fname in os.listdir(os.path.join(ROOT, "include")):
+        if not fname.endswith(".h"):
+            continue
+        src = open(os.path.join(ROOT, "include", fname)).read()
+        src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+        names += re.findall(r"^\s*(?:const\s+)?[A-Za-z_][A-Za-z0-9_]*\s*\*?\s*(dptq_[a-z0-9_]+)\s*\(", src, flags=re.M)
+    return sorted(set(names))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for required in ("dptq_pack_weights", "dptq_rotate_quant_act", "dptq_qlinear"):
+        assert required in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    from paper_2606_12487_gb300 import dptq
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+        assert name in dptq.EXPORTS, f"binding lacks {name}"
+
+
+def test_library_is_built_for_sm103a():
+    from paper_2606_12487_gb300 import build
+    assert "arch=compute_103a,code=sm_103a" in build.ARCH
+    assert os.path.exists(build.LIB)
+
+
+def test_status_strings(lib):
+    assert lib.dptq_status_str(0) == b"ok"
+    assert lib.dptq_status_str(5) == b"device wait timed out"
+
+
+def test_argument_checks_need_no_gpu(lib):
+    P = ctypes.c_void_p
+    dummy = P(16)
+    h = P()
+    # bits outside {4, 8}
+    assert lib.dptq_rotate_quant_act(dummy, 4, 256, 256, 5, dummy, dummy, None) == 1
+    assert b"bits" in lib.dptq_last_error_message()
+    # K not a multiple of 32 / bad Hadamard layout / null pointers / sizes
+    assert lib.dptq_rotate_quant_act(dummy, 4, 100, 64, 4, dummy, dummy, None) == 2
+    assert lib.dptq_rotate_quant_act(dummy, 4, 1536 + 96, 512, 4, dummy, dummy, None) == 2
+    assert lib.dptq_rotate_quant_act(None, 4, 256, 256, 4, dummy, dummy, None) == 1
+    assert lib.dptq_rotate_quant_act(dummy, -1, 256, 256, 4, dummy, dummy, None) == 1
+    assert lib.dptq_rotate_quant_act(dummy, 0, 256, 256, 4, dummy, dummy, None) == 0   # M == 0: no-op
+    assert lib.dptq_pack_weights(None, 16, 256, 256, 1, ctypes.byref(h)) == 1
+    assert lib.dptq_pack_weights(dummy, 0, 256, 256, 1, ctypes.byref(h)) == 1
+    assert lib.dptq_pack_weights(dummy, 24, 256, 256, 1, ctypes.byref(h)) == 2          # N % 16
+    assert lib.dptq_qlinear(None, dummy, 4, 4, dummy, None) == 1
+    assert lib.dptq_qlinear(None, dummy, 4, 3, dummy, None) == 1
+    assert lib.dptq_get_shape(None, None, None, None) == 1
+    lib.dptq_destroy(None)
+
+
+def test_binding_has_no_cpu_fallback():
+    # The binding forwards to the library only; it contains no compute path of its own.
+    src = open(os.path.join(ROOT, "paper_2606_12487_gb300", "dptq.py")).read()
+    assert "import oracle" not in src and "from oracle" not in src
+    for banned in ("numpy.matmul", "torch.matmul", "@ ", "hadamard"):
+        assert banned not in src
