@@ -33,8 +33,9 @@
  *     Online calls are asynchronous and stream-ordered; they do not synchronize the
  *     host.  Calls that share one handle, or the library scratch of one device,
  *     must not run concurrently on different streams.
- *   - Shape rules: 1 <= K, K % 32 == 0, N % 16 == 0, K splits into blocks of
- *     had_block plus a power-of-two tail, bits in {4, 8}.  Violations return
+ *   - Shape rules: 1 <= K <= 49152, K % 32 == 0, N % 16 == 0, had_block a power of
+ *     two <= 4096, K splits into blocks of had_block plus a power-of-two tail, bits in
+ *     {4, 8}.  Violations return
  *     DPTQ_ERR_INVALID_ARG (bits, null pointers, negative sizes) or
  *     DPTQ_ERR_UNSUPPORTED (shape).  M == 0 is a no-op.
  *   - No exception crosses this boundary.  CUDA errors map to DPTQ_ERR_CUDA; the
@@ -84,8 +85,8 @@ dptq_status dptq_pack_weights(const void* W_fp16, int N, int K, int had_block, i
  *   bits 0-3 and code 2j+1 in bits 4-7, each 4-bit two's complement;
  *   bits == 8: int8 [M][K].
  * scales (device, written): float [M], s_a per token.
- * One fused kernel: 128-bit loads, Walsh-Hadamard butterflies in fp32, row absmax,
- * rounding, packing. */
+ * One fused kernel: 128-bit loads, Walsh-Hadamard butterflies on exact 64-bit fixed
+ * point, one correctly rounded conversion to fp32, row absmax, rounding, packing. */
 dptq_status dptq_rotate_quant_act(const void* x_fp16, int M, int K, int had_block, int bits,
                                   void* codes, float* scales, void* stream);
 

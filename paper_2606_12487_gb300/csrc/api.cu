@@ -65,6 +65,7 @@ int rq_chunk(int K, int B) {
 
 dptq_status check_shape(int K, int B, int& nfull, int& tail, int& log2B) {
   if (K % 32 != 0) return fail(DPTQ_ERR_UNSUPPORTED, "K must be a multiple of 32");
+  if (B > 4096) return fail(DPTQ_ERR_UNSUPPORTED, "had_block above 4096 is not supported");
   if (!hadamard_layout(K, B, nfull, tail, log2B))
     return fail(DPTQ_ERR_UNSUPPORTED, "K must split into blocks of had_block (a power of two) plus a power-of-two tail");
   if (rotate_quant_smem(K, rq_chunk(K, B)) > kSmemPerBlock)
@@ -222,7 +223,7 @@ dptq_status dptq_pack_weights(const void* W_fp16, int N, int K, int had_block, i
   h->device = dev;
   h->N = N;
   h->K = K;
-  h->K_pad = round_up(K, kKBlock);
+  h->K_pad = round_up(K, kKPad);
   h->KB = h->K_pad / kKBlock;
   h->N_pad = round_up(N, 128);
   h->had_block = had_block;

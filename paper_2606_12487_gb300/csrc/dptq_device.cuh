@@ -64,6 +64,7 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
   const long long t0 = clock64();
   while (true) {
     if (mbar_try_wait(bar, parity)) return true;
+    __nanosleep(20);   // yield issue slots to the warps doing work
     if (*abort_flag) return false;
     if (clock64() - t0 > kWaitTimeoutCycles) {
       *abort_flag = 1;

@@ -8,8 +8,10 @@
 namespace dptq {
 
 // K is processed in blocks of 128 elements: one 128-byte row of the MMA's swizzled
-// FP8 operand tile.
+// FP8 operand tile.  Packed weights and activation operands pad K to a multiple of
+// kKPad so that a pipeline stage may hold two blocks.
 constexpr int kKBlock = 128;
+constexpr int kKPad = 256;
 // One (128 output channels) x (128 k) tile of packed 4-bit weights.
 constexpr int kWTileBytes = 128 * 64;
 
@@ -67,19 +69,21 @@ struct GemmArgs {
   uint32_t* counters;  // [grid] arrival counters (zero between launches)
   int* err;            // device error word
   int M, N, M_pad, KB, planes;
+  int KI;              // pipeline iterations per tile (KB / k-blocks per stage)
   int n_wtiles;        // N_pad / 128
   int m_tiles;         // M_pad / NT
-  int seg_blocks;      // k-blocks per exact fp32 accumulation segment
+  int seg_iters;       // iterations per exact fp32 accumulation segment
   int segs;            // accumulator segments per tile
   int nbuf;            // TMEM accumulator buffers (1 or 2)
   int stages;          // shared-memory pipeline depth
   int dp_tiles;        // tiles processed whole, round-robin, before the stream-K part
-  long long sk_iters;  // stream-K iterations (tiles after dp_tiles, times KB)
+  long long sk_iters;  // stream-K iterations (tiles after dp_tiles, times KI)
   uint32_t tmem_cols;
 };
 
 struct GemmPlan {
   int nt;          // token tile (MMA N): 16, 32, 64, 128 or 256
+  int kps;         // k-blocks of 128 per pipeline stage (1 or 2)
   int M_pad;
   int grid;
   int smem_bytes;

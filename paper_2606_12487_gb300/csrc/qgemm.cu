@@ -22,10 +22,11 @@
 //
 // Warp roles of the persistent CTA (one per SM):
 //   warp 0      producer: bulk copies (TMA engine) of packed weight tiles and of the
-//               pre-swizzled E4M3 activation tiles into a `stages`-deep ring
+//               pre-swizzled E4M3 activation tiles into a `stages`-deep ring; a stage
+//               holds KPS k-blocks of 128
 //   warp 1      TMEM allocator + single-thread tcgen05.mma issuer
-//   warps 2-5   converters: packed int4 -> E4M3 in the 128-byte swizzle layout
-//   warps 6-9   epilogue: tcgen05.ld -> int32 -> scales -> fp16, or int32 atomics into
+//   warps 2-9   converters: packed int4 -> E4M3 in the 128-byte swizzle layout
+//   warps 10-13 epilogue: tcgen05.ld -> int32 -> scales -> fp16, or int32 atomics into
 //               the split-tile scratch, the last contributor finishing the tile
 // Work: whole tiles round-robin first (`dp_tiles`), then the remaining tiles' k-blocks
 // split evenly over the CTAs (stream-K), so every SM streams the same number of
@@ -39,9 +40,10 @@
 
 namespace dptq {
 
-constexpr int kGemmThreads = 320;
-constexpr int kConvWarp0 = 2, kNumConvWarps = 4;
-constexpr int kEpiWarp0 = 6, kNumEpiWarps = 4;
+constexpr int kNumConvWarps = 8, kConvWarp0 = 2;
+constexpr int kNumEpiWarps = 4, kEpiWarp0 = kConvWarp0 + kNumConvWarps;
+constexpr int kGemmThreads = 32 * (kEpiWarp0 + kNumEpiWarps);   // 448
+constexpr int kConvThreads = 32 * kNumConvWarps;
 constexpr int kConvBytes = 128 * 128;   // one weight tile widened to E4M3
 constexpr int kMaxStages = 8;
 constexpr int kSmemLimit = 232448;      // 227 KB opt-in dynamic shared memory per CTA
@@ -49,14 +51,14 @@ constexpr int kBarrierBytes = 1024;
 
 struct Unit {
   int tile;
-  int kb0, kb1;
+  int i0, i1;        // iteration range (stages of KPS k-blocks) within the tile
   int slot;          // split-tile scratch slot, -1 when this CTA owns the whole tile
   int contributors;  // CTAs that add into the slot
 };
 
 // Deterministic enumeration of one CTA's work; every warp role walks the same list.
 struct UnitIter {
-  int cta, G, KB, dp_tiles, dp_next;
+  int cta, G, KI, dp_tiles, dp_next;
   long long sk_iters, it, it_end;
 
   __device__ __forceinline__ long long sk_begin(int c) const { return ((long long)c * sk_iters) / G; }
@@ -66,7 +68,7 @@ struct UnitIter {
   __device__ __forceinline__ void init(const GemmArgs& a) {
     cta = blockIdx.x;
     G = gridDim.x;
-    KB = a.KB;
+    KI = a.KI;
     dp_tiles = a.dp_tiles;
     dp_next = cta;
     sk_iters = a.sk_iters;
@@ -76,26 +78,41 @@ struct UnitIter {
   __device__ __forceinline__ bool next(Unit& u) {
     if (dp_next < dp_tiles) {
       u.tile = dp_next;
-      u.kb0 = 0;
-      u.kb1 = KB;
+      u.i0 = 0;
+      u.i1 = KI;
       u.slot = -1;
       u.contributors = 1;
       dp_next += G;
       return true;
     }
     if (it >= it_end) return false;
-    const long long t = it / KB;
-    const int kb0 = (int)(it - t * KB);
+    const long long t = it / KI;
+    const int i0 = (int)(it - t * KI);
     const long long left = it_end - it;
-    const int kb1 = (int)((long long)(KB - kb0) < left ? KB : kb0 + left);
-    const int c0 = cta_of(t * KB), c1 = cta_of(t * KB + KB - 1);
+    const int i1 = (int)((long long)(KI - i0) < left ? KI : i0 + left);
+    const int c0 = cta_of(t * KI), c1 = cta_of(t * KI + KI - 1);
     u.tile = dp_tiles + (int)t;
-    u.kb0 = kb0;
-    u.kb1 = kb1;
+    u.i0 = i0;
+    u.i1 = i1;
     u.slot = (c0 == c1) ? -1 : c0;
     u.contributors = c1 - c0 + 1;
-    it += kb1 - kb0;
+    it += i1 - i0;
     return true;
+  }
+};
+
+// Ring position (stage index and the parity of its current phase), advanced without
+// divisions.
+struct Ring {
+  int s = 0;
+  uint32_t ph = 0;
+  int S;
+  __device__ __forceinline__ explicit Ring(int stages) : S(stages) {}
+  __device__ __forceinline__ void next() {
+    if (++s == S) {
+      s = 0;
+      ph ^= 1u;
+    }
   }
 };
 
@@ -108,24 +125,33 @@ __device__ __forceinline__ uint32_t widen_hi(uint32_t w) {
   return ((w >> 4) & 0x07070707u) | (w & 0x80808080u);
 }
 
-template <int NT>
+// Shared-memory layout of one pipeline stage: KPS widened weight tiles (1024-aligned
+// swizzle atoms), KPS x planes token tiles, then the KPS packed weight tiles.
+template <int NT, int KPS>
 struct Smem {
-  static constexpr int kActBytes = NT * 128;  // one plane of the token tile
+  static constexpr int kActBytes = NT * 128;  // one plane of one token tile
   uint8_t* base;
-  int stages, planes;
-  __device__ __forceinline__ int stage_bytes() const { return kConvBytes + planes * kActBytes + kWTileBytes; }
-  __device__ __forceinline__ uint8_t* conv(int s) const { return base + s * stage_bytes(); }
-  __device__ __forceinline__ uint8_t* act(int s, int p) const { return conv(s) + kConvBytes + p * kActBytes; }
-  __device__ __forceinline__ uint8_t* wpack(int s) const { return conv(s) + kConvBytes + planes * kActBytes; }
+  int planes;
+  int stage_bytes;
+  __device__ __forceinline__ Smem(uint8_t* b, int p) : base(b), planes(p) {
+    stage_bytes = KPS * (kConvBytes + p * kActBytes + kWTileBytes);
+  }
+  __device__ __forceinline__ uint8_t* conv(int s, int h) const { return base + s * stage_bytes + h * kConvBytes; }
+  __device__ __forceinline__ uint8_t* act(int s, int h, int p) const {
+    return base + s * stage_bytes + KPS * kConvBytes + (h * planes + p) * kActBytes;
+  }
+  __device__ __forceinline__ uint8_t* wpack(int s) const {
+    return base + s * stage_bytes + KPS * (kConvBytes + planes * kActBytes);
+  }
 };
 
-template <int NT>
+template <int NT, int KPS>
 __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int S = a.stages;
-  Smem<NT> sm{smem, S, a.planes};
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + S * sm.stage_bytes());
+  const Smem<NT, KPS> sm(smem, a.planes);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + S * sm.stage_bytes);
   uint64_t* full = bars;
   uint64_t* convb = bars + kMaxStages;
   uint64_t* empty = bars + 2 * kMaxStages;
@@ -136,6 +162,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
   uint32_t* tmem_base_sh = reinterpret_cast<uint32_t*>(esync + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_base_sh + 1);
   volatile int* last_flag = reinterpret_cast<volatile int*>(tmem_base_sh + 2);
+  const uint8_t** pend_src = reinterpret_cast<const uint8_t**>(tmem_base_sh + 8);   // producer's pending list
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -176,38 +203,42 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
       const uint64_t pol_w = l2_policy_evict_first();   // weights are streamed once
       const uint64_t pol_a = l2_policy_evict_last();    // activations are re-read per n-tile
       const uint32_t act_bytes = (uint32_t)NT * 128;
-      const uint32_t tx = (uint32_t)kWTileBytes + (uint32_t)a.planes * act_bytes;
+      const uint32_t w_bytes = (uint32_t)KPS * kWTileBytes;
+      const uint32_t tx = w_bytes + (uint32_t)(KPS * a.planes) * act_bytes;
       const size_t plane_stride = (size_t)a.KB * a.M_pad * 128;
+      const size_t kb_stride = (size_t)a.M_pad * 128;
       // Weight tiles do not depend on the previous kernel; the first `S` stages are
       // requested before waiting for it (programmatic dependent launch) and their
       // activation halves are issued once the previous kernel has finished.
       bool waited = false;
       int npend = 0;
-      int pend_s[kMaxStages];
-      const uint8_t* pend_src[kMaxStages];
+      Ring rg(S);
       int g = 0;
       while (iter.next(un)) {
         const int nt = un.tile / a.m_tiles;
         const int mt = un.tile - nt * a.m_tiles;
-        for (int kb = un.kb0; kb < un.kb1; ++kb, ++g) {
-          const int s = g % S;
-          if (!mbar_wait(&empty[s], ((g / S) & 1) ^ 1, abort_flag, a.err, kDevTimeoutEmpty)) goto producer_done;
+        const uint8_t* wsrc = a.wt + ((size_t)nt * a.KB + (size_t)un.i0 * KPS) * kWTileBytes;
+        const uint8_t* asrc = a.act + ((size_t)un.i0 * KPS * a.M_pad + (size_t)mt * NT) * 128;
+        for (int it = un.i0; it < un.i1; ++it, ++g, rg.next(), wsrc += w_bytes, asrc += KPS * kb_stride) {
+          const int s = rg.s;
+          if (!mbar_wait(&empty[s], rg.ph ^ 1u, abort_flag, a.err, kDevTimeoutEmpty)) goto producer_done;
           mbar_arrive_expect_tx(&full[s], tx);
-          bulk_g2s(sm.wpack(s), a.wt + ((size_t)nt * a.KB + kb) * kWTileBytes, kWTileBytes, &full[s], pol_w);
-          const uint8_t* asrc = a.act + ((size_t)kb * a.M_pad + (size_t)mt * NT) * 128;
+          bulk_g2s(sm.wpack(s), wsrc, w_bytes, &full[s], pol_w);
           if (waited) {
-            for (int p = 0; p < a.planes; ++p)
-              bulk_g2s(sm.act(s, p), asrc + p * plane_stride, act_bytes, &full[s], pol_a);
+#pragma unroll
+            for (int h = 0; h < KPS; ++h)
+              for (int p = 0; p < a.planes; ++p)
+                bulk_g2s(sm.act(s, h, p), asrc + h * kb_stride + p * plane_stride, act_bytes, &full[s], pol_a);
           } else {
-            pend_s[npend] = s;
-            pend_src[npend] = asrc;
-            ++npend;
+            pend_src[npend++] = asrc;   // stage index of pending entry i is i
             if (npend == S) {
               pdl_wait();
               waited = true;
               for (int i = 0; i < npend; ++i)
-                for (int p = 0; p < a.planes; ++p)
-                  bulk_g2s(sm.act(pend_s[i], p), pend_src[i] + p * plane_stride, act_bytes, &full[pend_s[i]], pol_a);
+                for (int h = 0; h < KPS; ++h)
+                  for (int p = 0; p < a.planes; ++p)
+                    bulk_g2s(sm.act(i, h, p), pend_src[i] + h * kb_stride + p * plane_stride, act_bytes,
+                             &full[i], pol_a);
               npend = 0;
             }
           }
@@ -216,8 +247,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
       if (!waited) {
         pdl_wait();
         for (int i = 0; i < npend; ++i)
-          for (int p = 0; p < a.planes; ++p)
-            bulk_g2s(sm.act(pend_s[i], p), pend_src[i] + p * plane_stride, act_bytes, &full[pend_s[i]], pol_a);
+          for (int h = 0; h < KPS; ++h)
+            for (int p = 0; p < a.planes; ++p)
+              bulk_g2s(sm.act(i, h, p), pend_src[i] + h * kb_stride + p * plane_stride, act_bytes, &full[i], pol_a);
       }
     producer_done:
       // Do not leave the CTA while copies into its shared memory may be in flight.
@@ -231,30 +263,34 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
       const uint32_t idesc = idesc_e4m3_m128(NT);
-      int g = 0, u = 0;
+      Ring rg(S);
+      int u = 0;
       while (iter.next(un)) {
         const int b = a.nbuf == 2 ? (u & 1) : 0;
         const uint32_t tpar = ((a.nbuf == 2 ? (u >> 1) : u) & 1) ^ 1;
         if (!mbar_wait(&tempty[b], tpar, abort_flag, a.err, kDevTimeoutTmemEmpty)) break;
         tc_fence_after();
         const uint32_t dbase = tmem_base + (uint32_t)(b * NT * a.segs);
-        const int seg0 = un.kb0 / a.seg_blocks;
+        const int seg0 = un.i0 / a.seg_iters;
         bool ok = true;
-        for (int kb = un.kb0; kb < un.kb1; ++kb, ++g) {
-          const int s = g % S;
-          if (!mbar_wait(&convb[s], (g / S) & 1, abort_flag, a.err, kDevTimeoutConv)) {
+        for (int it = un.i0; it < un.i1; ++it, rg.next()) {
+          const int s = rg.s;
+          if (!mbar_wait(&convb[s], rg.ph, abort_flag, a.err, kDevTimeoutConv)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t d = dbase + (uint32_t)((kb / a.seg_blocks - seg0) * NT);
-          const bool fresh = (kb == un.kb0) || (kb % a.seg_blocks == 0);
-          const uint64_t ad = sdesc_sw128(smem_u32(sm.conv(s)));
-          for (int p = 0; p < a.planes; ++p) {
-            const uint64_t bd = sdesc_sw128(smem_u32(sm.act(s, p)));
+          const uint32_t d = dbase + (uint32_t)((it / a.seg_iters - seg0) * NT);
+          const bool fresh = (it == un.i0) || (it % a.seg_iters == 0);
 #pragma unroll
-            for (int ks = 0; ks < 4; ++ks)   // 4 x (K = 32 FP8 elements = 32 bytes)
-              mma_f8(d, ad + 2 * ks, bd + 2 * ks, idesc, (fresh && p == 0 && ks == 0) ? 0u : 1u);
+          for (int h = 0; h < KPS; ++h) {
+            const uint64_t ad = sdesc_sw128(smem_u32(sm.conv(s, h)));
+            for (int p = 0; p < a.planes; ++p) {
+              const uint64_t bd = sdesc_sw128(smem_u32(sm.act(s, h, p)));
+#pragma unroll
+              for (int ks = 0; ks < 4; ++ks)   // 4 x (K = 32 FP8 elements = 32 bytes)
+                mma_f8(d, ad + 2 * ks, bd + 2 * ks, idesc, (fresh && h == 0 && p == 0 && ks == 0) ? 0u : 1u);
+            }
           }
           mma_commit(&empty[s]);
         }
@@ -269,25 +305,35 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
     }
   } else if (warp < kEpiWarp0) {
     // ------------------------------------------------------------ converters
-    const int ctid = threadIdx.x - kConvWarp0 * 32;   // 0..127
-    int g = 0;
+    const int ctid = threadIdx.x - kConvWarp0 * 32;   // 0..255
+    Ring rg(S);
     while (iter.next(un)) {
       bool ok = true;
-      for (int kb = un.kb0; kb < un.kb1; ++kb, ++g) {
-        const int s = g % S;
-        if (!mbar_wait(&full[s], (g / S) & 1, abort_flag, a.err, kDevTimeoutFull)) {
+      for (int it = un.i0; it < un.i1; ++it, rg.next()) {
+        const int s = rg.s;
+        if (!mbar_wait(&full[s], rg.ph, abort_flag, a.err, kDevTimeoutFull)) {
           ok = false;
           break;
         }
-        const uint8_t* wp = sm.wpack(s);
-        uint8_t* cv = sm.conv(s);
+        const uint8_t* __restrict__ wp = sm.wpack(s);
+        // Each thread widens 2 * KPS x 16 packed bytes: (tile h, row r, chunks j0 and
+        // j0 + 1) of 16 weights each.  All loads are issued before any store.
+        uint4 w[2 * KPS];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          const int unit = i * 128 + ctid;   // (row r, 16-weight chunk j)
-          const int r = unit >> 3, j = unit & 7;
-          const uint2 w = *reinterpret_cast<const uint2*>(wp + r * 64 + j * 8);
-          const uint4 o = make_uint4(widen_lo(w.x), widen_hi(w.x), widen_lo(w.y), widen_hi(w.y));
-          *reinterpret_cast<uint4*>(cv + r * 128 + ((j ^ (r & 7)) << 4)) = o;
+        for (int i = 0; i < 2 * KPS; ++i) {
+          const int p = i * kConvThreads + ctid;   // 16-byte unit: tile p >> 9
+          w[i] = *reinterpret_cast<const uint4*>(wp + (p >> 9) * kWTileBytes + ((p & 511) >> 2) * 64 + (p & 3) * 16);
+        }
+#pragma unroll
+        for (int i = 0; i < 2 * KPS; ++i) {
+          const int p = i * kConvThreads + ctid;
+          const int q = p & 511;
+          const int r = q >> 2, j0 = (q & 3) * 2;
+          uint8_t* row = sm.conv(s, p >> 9) + r * 128;
+          *reinterpret_cast<uint4*>(row + ((j0 ^ (r & 7)) << 4)) =
+              make_uint4(widen_lo(w[i].x), widen_hi(w[i].x), widen_lo(w[i].y), widen_hi(w[i].y));
+          *reinterpret_cast<uint4*>(row + (((j0 + 1) ^ (r & 7)) << 4)) =
+              make_uint4(widen_lo(w[i].z), widen_hi(w[i].z), widen_lo(w[i].w), widen_hi(w[i].w));
         }
         fence_proxy_async_smem();
         __syncwarp();
@@ -298,6 +344,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
   } else {
     // ------------------------------------------------------------ epilogue
     pdl_wait();   // scales come from the previous kernel; `out` may still be read by it
+    const float* __restrict__ sa_g = a.sa;
+    const float* __restrict__ sw_g = a.sw;
+    __half* __restrict__ out_g = a.out;
+    int32_t* __restrict__ acc_g = a.acc_out;
+    int32_t* __restrict__ ws_g = a.ws;
     const int q = warp & 3;                    // TMEM lane quarter of this warp
     const int etid = threadIdx.x - kEpiWarp0 * 32;
     const uint32_t lane_base = (uint32_t)(q * 32) << 16;
@@ -321,10 +372,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
       const int mt = un.tile - nt * a.m_tiles;
       const int n = nt * 128 + q * 32 + lane;
       const int m0 = mt * NT;
-      const int nseg = (un.kb1 - 1) / a.seg_blocks - un.kb0 / a.seg_blocks + 1;
+      const int nseg = (un.i1 - 1) / a.seg_iters - un.i0 / a.seg_iters + 1;
       const uint32_t tb = tmem_base + lane_base + (uint32_t)(b * NT * a.segs);
-      const float swn = n < a.N ? a.sw[n] : 0.f;
-      int32_t* wsl = un.slot >= 0 ? a.ws + (size_t)un.slot * (NT * 128) : nullptr;
+      const float swn = n < a.N ? sw_g[n] : 0.f;
+      int32_t* __restrict__ wsl = un.slot >= 0 ? ws_g + (size_t)un.slot * (NT * 128) : nullptr;
 #pragma unroll 1
       for (int c0 = 0; c0 < NT; c0 += 16) {
         int acc[16];
@@ -338,14 +389,17 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
           for (int i = 0; i < 16; ++i) acc[i] += __float2int_rn(__uint_as_float(r[i]) * 512.f);
         }
         if (wsl == nullptr) {
+          float sav[16];
+#pragma unroll
+          for (int i = 0; i < 16; ++i) sav[i] = (m0 + c0 + i < a.M) ? sa_g[m0 + c0 + i] : 0.f;
           if (n < a.N) {
 #pragma unroll
             for (int i = 0; i < 16; ++i) {
               const int m = m0 + c0 + i;
               if (m < a.M) {
-                const float t = __fmul_rn(__int2float_rn(acc[i]), a.sa[m]);
-                a.out[(size_t)m * a.N + n] = __float2half_rn(__fmul_rn(t, swn));
-                if (a.acc_out) a.acc_out[(size_t)m * a.N + n] = acc[i];
+                const float t = __fmul_rn(__int2float_rn(acc[i]), sav[i]);
+                out_g[(size_t)m * a.N + n] = __float2half_rn(__fmul_rn(t, swn));
+                if (acc_g) acc_g[(size_t)m * a.N + n] = acc[i];
               }
             }
           }
@@ -371,15 +425,26 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
         if (!epi_sync()) break;
         if (*last_flag) {
           __threadfence();
-          for (int c = 0; c < NT; ++c) {
-            int32_t* p = wsl + c * 128 + q * 32 + lane;
-            const int v = __ldcg(p);
-            __stcg(p, 0);   // leave the scratch zeroed for the next launch
-            const int m = m0 + c;
-            if (n < a.N && m < a.M) {
-              const float t = __fmul_rn(__int2float_rn(v), a.sa[m]);
-              a.out[(size_t)m * a.N + n] = __float2half_rn(__fmul_rn(t, swn));
-              if (a.acc_out) a.acc_out[(size_t)m * a.N + n] = v;
+#pragma unroll 1
+          for (int c0 = 0; c0 < NT; c0 += 16) {
+            int v[16];
+            float sav[16];
+#pragma unroll
+            for (int i = 0; i < 16; ++i) v[i] = __ldcg(wsl + (c0 + i) * 128 + q * 32 + lane);
+#pragma unroll
+            for (int i = 0; i < 16; ++i) sav[i] = (m0 + c0 + i < a.M) ? sa_g[m0 + c0 + i] : 0.f;
+#pragma unroll
+            for (int i = 0; i < 16; ++i) __stcg(wsl + (c0 + i) * 128 + q * 32 + lane, 0);   // zeroed for the next launch
+            if (n < a.N) {
+#pragma unroll
+              for (int i = 0; i < 16; ++i) {
+                const int m = m0 + c0 + i;
+                if (m < a.M) {
+                  const float t = __fmul_rn(__int2float_rn(v[i]), sav[i]);
+                  out_g[(size_t)m * a.N + n] = __float2half_rn(__fmul_rn(t, swn));
+                  if (acc_g) acc_g[(size_t)m * a.N + n] = v[i];
+                }
+              }
             }
           }
         }
@@ -406,75 +471,86 @@ int gemm_pick_nt(int M, int bits, int KB) {
   return 256;
 }
 
-template <int NT>
-static int gemm_smem_bytes(int stages, int planes) {
-  return 1024 + stages * (kConvBytes + planes * NT * 128 + kWTileBytes) + kBarrierBytes;
-}
+// Token tiles of up to 64 columns stream weights (decode): two k-blocks per stage to
+// halve the per-byte barrier and conversion overhead.  Wider tiles are MMA-bound and
+// keep one k-block per stage for a deeper ring.
+static int kps_for(int nt) { return nt <= 64 ? 2 : 1; }
 
-static int smem_for(int nt, int stages, int planes) {
-  switch (nt) {
-    case 16: return gemm_smem_bytes<16>(stages, planes);
-    case 32: return gemm_smem_bytes<32>(stages, planes);
-    case 64: return gemm_smem_bytes<64>(stages, planes);
-    case 128: return gemm_smem_bytes<128>(stages, planes);
-    default: return gemm_smem_bytes<256>(stages, planes);
-  }
+static int smem_for(int nt, int kps, int stages, int planes) {
+  return 1024 + stages * kps * (kConvBytes + planes * nt * 128 + kWTileBytes) + kBarrierBytes;
 }
 
 bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan) {
   GemmArgs& a = plan.args;
   const int KB = K_pad / kKBlock;
   const int planes = bits == 8 ? 2 : 1;
-  // Largest |code| * |weight| per k-block, and the k-blocks one fp32 accumulator can
-  // take before the exact-integer bound 2^24 could be crossed.
-  const long long per_block = (long long)(bits == 8 ? 128 : 8) * 7 * kKBlock;
-  int seg_blocks = (int)(((1LL << 24) - 1) / per_block);
-  if (seg_blocks > KB) seg_blocks = KB;
-  const int segs = ceil_div(KB, seg_blocks);
   int nt = gemm_pick_nt(M, bits, KB);
-  while (nt > 16 && nt * segs > 512) nt >>= 1;
+  int kps = kps_for(nt);
+  if (KB % kps != 0) kps = 1;
+  // Largest |code| * |weight| sum per stage, and the stages one fp32 accumulator can
+  // take before the exact-integer bound 2^24 could be crossed.
+  auto seg_plan = [&](int kps_, int& seg_iters, int& segs) {
+    const int KI = KB / kps_;
+    const long long per_iter = (long long)(bits == 8 ? 128 : 8) * 7 * kKBlock * kps_;
+    seg_iters = (int)(((1LL << 24) - 1) / per_iter);
+    if (seg_iters > KI) seg_iters = KI;
+    segs = (KI + seg_iters - 1) / seg_iters;
+  };
+  int seg_iters, segs;
+  seg_plan(kps, seg_iters, segs);
+  while (nt > 16 && nt * segs > 512) {
+    nt >>= 1;
+    if (kps_for(nt) != kps && KB % kps_for(nt) == 0) {
+      kps = kps_for(nt);
+      seg_plan(kps, seg_iters, segs);
+    }
+  }
   if (nt * segs > 512) return false;
   int stages = kMaxStages;
-  while (stages > 2 && smem_for(nt, stages, planes) > kSmemLimit) --stages;
-  if (smem_for(nt, stages, planes) > kSmemLimit) return false;
+  while (stages > 2 && smem_for(nt, kps, stages, planes) > kSmemLimit) --stages;
+  if (smem_for(nt, kps, stages, planes) > kSmemLimit) return false;
   const int nbuf = 2 * nt * segs <= 512 ? 2 : 1;
   uint32_t cols = 32;
   while (cols < (uint32_t)(nbuf * nt * segs)) cols <<= 1;
 
+  const int KI = KB / kps;
   const int M_pad = round_up(M, nt);
   const int n_wtiles = ceil_div(N, 128);
   const int m_tiles = M_pad / nt;
   const long long tiles = (long long)n_wtiles * m_tiles;
-  const long long iters = tiles * KB;
+  const long long iters = tiles * KI;
   int G = (int)(iters < num_sms ? iters : num_sms);
   if (G < 1) G = 1;
   long long dp = 0;
   if (tiles >= 2LL * G) dp = (tiles / G - 1) * G;
 
   plan.nt = nt;
+  plan.kps = kps;
   plan.M_pad = M_pad;
   plan.grid = G;
-  plan.smem_bytes = smem_for(nt, stages, planes);
+  plan.smem_bytes = smem_for(nt, kps, stages, planes);
   a.M = M;
   a.N = N;
   a.M_pad = M_pad;
   a.KB = KB;
+  a.KI = KI;
   a.planes = planes;
   a.n_wtiles = n_wtiles;
   a.m_tiles = m_tiles;
-  a.seg_blocks = seg_blocks;
+  a.seg_iters = seg_iters;
   a.segs = segs;
   a.nbuf = nbuf;
   a.stages = stages;
   a.dp_tiles = (int)dp;
-  a.sk_iters = (tiles - dp) * KB;
+  a.sk_iters = (tiles - dp) * KI;
   a.tmem_cols = cols;
   return true;
 }
 
-template <int NT>
+template <int NT, int KPS>
 static cudaError_t launch_nt(const GemmPlan& plan, cudaStream_t s, bool pdl) {
-  cudaError_t e = cudaFuncSetAttribute(qgemm_kernel<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize, plan.smem_bytes);
+  cudaError_t e =
+      cudaFuncSetAttribute(qgemm_kernel<NT, KPS>, cudaFuncAttributeMaxDynamicSharedMemorySize, plan.smem_bytes);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)plan.grid);
@@ -486,16 +562,24 @@ static cudaError_t launch_nt(const GemmPlan& plan, cudaStream_t s, bool pdl) {
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
-  return cudaLaunchKernelEx(&cfg, qgemm_kernel<NT>, plan.args);
+  return cudaLaunchKernelEx(&cfg, qgemm_kernel<NT, KPS>, plan.args);
 }
 
 cudaError_t launch_gemm(const GemmPlan& plan, cudaStream_t s, bool pdl) {
+  if (plan.kps == 2) {
+    switch (plan.nt) {
+      case 16: return launch_nt<16, 2>(plan, s, pdl);
+      case 32: return launch_nt<32, 2>(plan, s, pdl);
+      case 64: return launch_nt<64, 2>(plan, s, pdl);
+      default: return cudaErrorInvalidValue;
+    }
+  }
   switch (plan.nt) {
-    case 16: return launch_nt<16>(plan, s, pdl);
-    case 32: return launch_nt<32>(plan, s, pdl);
-    case 64: return launch_nt<64>(plan, s, pdl);
-    case 128: return launch_nt<128>(plan, s, pdl);
-    case 256: return launch_nt<256>(plan, s, pdl);
+    case 16: return launch_nt<16, 1>(plan, s, pdl);
+    case 32: return launch_nt<32, 1>(plan, s, pdl);
+    case 64: return launch_nt<64, 1>(plan, s, pdl);
+    case 128: return launch_nt<128, 1>(plan, s, pdl);
+    case 256: return launch_nt<256, 1>(plan, s, pdl);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -1,8 +1,8 @@
 // rotate_quant.cu -- fused online block-Hadamard rotation + symmetric per-row
 // quantization (Section 2, Eq. 4 then Eq. 2; Section 4.2 per-token / per-channel
-// symmetric).  One CTA per row: 128-bit loads of the fp16 row into shared memory,
-// Walsh-Hadamard butterflies per block (natural Sylvester order) on exact 64-bit
-// fixed-point values, one correctly rounded conversion to fp32 including 1/sqrt(block),
+// symmetric).  One CTA per row: 128-bit loads of the fp16 row, Walsh-Hadamard
+// butterflies per block (natural Sylvester order) on exact 64-bit fixed-point values
+// in registers with two shared-memory transposes per 4096-element chunk, one correctly rounded conversion to fp32 including 1/sqrt(block),
 // row absmax by warp shuffles, IEEE-division rounding to the
 // integer grid, and one of four writers:
 //   kRQPublic   public codes (A4 packed nibbles / A8 int8) + fp32 scales
@@ -76,11 +76,26 @@ __device__ __forceinline__ float fixed_to_rotated(long long S, int log2n, float 
   return __fmul_rn(__fadd_rn(p, t), scale);
 }
 
+// The row is rotated in chunks of 4096 elements (whole Hadamard blocks; the last chunk
+// may be shorter).  Thread t holds 16 values of a chunk at a time, as exact 64-bit
+// fixed point, in three rounds that each cover 4 bits of the element index:
+//   round A: i = 16 t + e          (butterfly strides 1, 2, 4, 8 inside the thread)
+//   round B: i = 256 (t>>4) + 16 e + (t&15)   (strides 16 .. 128)
+//   round C: i = 256 e + t                    (strides 256 .. 2048)
+// with two transposes through shared memory in between (rows of 16 values padded by
+// one slot, so every access pattern is free of bank conflicts).  A stride applies to an
+// element only while it is below the size of the element's Hadamard block (B, or the
+// row's tail block).
+constexpr int kChunk = 4096;
+constexpr int kChunkPadded = kChunk + kChunk / 16;
+
+__device__ __forceinline__ int pad_idx(int i) { return i + (i >> 4); }
+
 template <int MODE>
 __global__ void __launch_bounds__(kRQThreads) rotate_quant_kernel(const RQArgs a) {
   extern __shared__ __align__(16) unsigned char rq_smem[];
-  float* sy = reinterpret_cast<float*>(rq_smem);                                     // the row, K floats
-  long long* sx = reinterpret_cast<long long*>(rq_smem + (size_t)a.K * sizeof(float));  // chunk, fixed point
+  float* sy = reinterpret_cast<float*>(rq_smem);                                      // the row, K floats
+  long long* sx = reinterpret_cast<long long*>(rq_smem + (size_t)a.K * sizeof(float));  // one padded chunk
   __shared__ float red[kRQThreads / 32];
   pdl_launch_dependents();
   pdl_wait();
@@ -89,65 +104,107 @@ __global__ void __launch_bounds__(kRQThreads) rotate_quant_kernel(const RQArgs a
   const int tid = threadIdx.x;
   const int K = a.K;
   const bool live = row < a.rows_in;
+  const int tail_start = a.nfull << a.log2B;   // first element of the tail block
 
   if (live) {
-    // The row is rotated chunk by chunk (a chunk holds whole Hadamard blocks); within
-    // a chunk the butterflies run on exact 64-bit integers, so the only rounding of the
-    // rotation is the final conversion to fp32.
     const uint4* src = reinterpret_cast<const uint4*>(a.x + (size_t)row * K);
-    const int reg_stages = a.log2B < 3 ? a.log2B : 3;   // strides 1, 2, 4 inside a thread
-    for (int c0 = 0; c0 < K; c0 += a.chunk) {
-      const int len = min(a.chunk, K - c0);
-      __syncthreads();
-      for (int v = tid; v < len / 8; v += kRQThreads) {
-        const uint4 u = src[c0 / 8 + v];
-        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
-        long long f[8];
+    for (int c0 = 0; c0 < K; c0 += kChunk) {
+      const int len = min(kChunk, K - c0);
+      // log2 of the block size that element i of this chunk belongs to
+      auto lg = [&](int i) { return (c0 + i < tail_start) ? a.log2B : a.log2T; };
+      long long f[16];
+      // ---- round A: load 16 consecutive fp16 values
+      {
+        const int i0 = tid * 16;
+        if (i0 < len) {
+          const uint4 u0 = src[(c0 + i0) / 8];
+          const uint4 u1 = src[(c0 + i0) / 8 + 1];
+          const uint32_t w[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          f[2 * i] = half_to_fixed(w[i] & 0xFFFFu);
-          f[2 * i + 1] = half_to_fixed(w[i] >> 16);
+          for (int k = 0; k < 8; ++k) {
+            f[2 * k] = half_to_fixed(w[k] & 0xFFFFu);
+            f[2 * k + 1] = half_to_fixed(w[k] >> 16);
+          }
+        } else {
+#pragma unroll
+          for (int k = 0; k < 16; ++k) f[k] = 0;
         }
+        const int L = lg(i0 < len ? i0 : 0);
 #pragma unroll
-        for (int ls = 0; ls < 3; ++ls) {
-          if (ls < reg_stages) {
-            const int h = 1 << ls;
+        for (int bit = 0; bit < 4; ++bit) {
+          if (bit < L) {
+            const int h = 1 << bit;
 #pragma unroll
-            for (int i = 0; i < 8; ++i) {
-              if ((i & h) == 0) {
-                const long long p = f[i], q = f[i + h];
-                f[i] = p + q;
-                f[i + h] = p - q;
+            for (int e = 0; e < 16; ++e)
+              if ((e & h) == 0) {
+                const long long p = f[e], q = f[e + h];
+                f[e] = p + q;
+                f[e + h] = p - q;
               }
-            }
           }
         }
+      }
+      const int maxlg = (c0 + len > tail_start) ? max(a.log2B, a.log2T) : a.log2B;
+      const int iA = tid * 16;
+      if (maxlg > 4) {
+        // ---- transpose A -> B
+        __syncthreads();   // the previous chunk's readers are done with sx
 #pragma unroll
-        for (int i = 0; i < 8; ++i) sx[8 * v + i] = f[i];
-      }
-      // Remaining strides in shared memory.  Blocks of B tile the chunk, except that
-      // the row's tail block (size `tail`) ends the last chunk and stops at h == tail.
-      const int nbf = len / 2;
-      const int halfB_log = a.log2B - 1;
-      const int tail_blk = (a.nfull * a.B - c0) >> a.log2B;   // chunk-local index of the tail block
-      for (int lh = reg_stages; lh < a.log2B; ++lh) {
-        const int h = 1 << lh;
+        for (int e = 0; e < 16; ++e) sx[pad_idx(iA + e)] = f[e];
         __syncthreads();
-        for (int b = tid; b < nbf; b += kRQThreads) {
-          const int blk = b >> halfB_log;
-          if (blk == tail_blk && h >= a.tail) continue;
-          const int bb = b - (blk << halfB_log);
-          const int i = (blk << a.log2B) + ((bb >> lh) << (lh + 1)) + (bb & (h - 1));
-          const long long p = sx[i], q = sx[i + h];
-          sx[i] = p + q;
-          sx[i + h] = p - q;
+        const int iB = 256 * (tid >> 4) + (tid & 15);
+#pragma unroll
+        for (int e = 0; e < 16; ++e) f[e] = sx[pad_idx(iB + 16 * e)];
+        const int L = lg(iB);
+#pragma unroll
+        for (int bit = 4; bit < 8; ++bit) {
+          if (bit < L) {
+            const int h = 1 << (bit - 4);
+#pragma unroll
+            for (int e = 0; e < 16; ++e)
+              if ((e & h) == 0) {
+                const long long p = f[e], q = f[e + h];
+                f[e] = p + q;
+                f[e + h] = p - q;
+              }
+          }
         }
-      }
-      __syncthreads();
-      for (int j = tid; j < len; j += kRQThreads) {
-        const int k = c0 + j;
-        const int log2n = (k >> a.log2B) < a.nfull ? a.log2B : a.log2T;
-        sy[k] = fixed_to_rotated(sx[j], log2n, a.c_hi, a.c_lo);
+        if (maxlg > 8) {
+          // ---- transpose B -> C
+#pragma unroll
+          for (int e = 0; e < 16; ++e) sx[pad_idx(iB + 16 * e)] = f[e];
+          __syncthreads();
+#pragma unroll
+          for (int e = 0; e < 16; ++e) f[e] = sx[pad_idx(256 * e + tid)];
+#pragma unroll
+          for (int bit = 8; bit < 12; ++bit) {
+            const int h = 1 << (bit - 8);
+#pragma unroll
+            for (int e = 0; e < 16; ++e)
+              if ((e & h) == 0 && bit < lg(256 * e + tid)) {
+                const long long p = f[e], q = f[e + h];
+                f[e] = p + q;
+                f[e + h] = p - q;
+              }
+          }
+#pragma unroll
+          for (int e = 0; e < 16; ++e) {
+            const int i = 256 * e + tid;
+            if (i < len) sy[c0 + i] = fixed_to_rotated(f[e], lg(i), a.c_hi, a.c_lo);
+          }
+        } else {
+#pragma unroll
+          for (int e = 0; e < 16; ++e) {
+            const int i = iB + 16 * e;
+            if (i < len) sy[c0 + i] = fixed_to_rotated(f[e], lg(i), a.c_hi, a.c_lo);
+          }
+        }
+      } else {
+#pragma unroll
+        for (int e = 0; e < 16; ++e) {
+          const int i = iA + e;
+          if (i < len) sy[c0 + i] = fixed_to_rotated(f[e], lg(i), a.c_hi, a.c_lo);
+        }
       }
     }
     __syncthreads();
@@ -261,7 +318,10 @@ __global__ void __launch_bounds__(kRQThreads) rotate_quant_kernel(const RQArgs a
   }
 }
 
-size_t rotate_quant_smem(int K, int chunk) { return (size_t)K * sizeof(float) + (size_t)chunk * sizeof(long long); }
+size_t rotate_quant_smem(int K, int chunk) {
+  (void)chunk;
+  return (size_t)K * sizeof(float) + (size_t)kChunkPadded * sizeof(long long);
+}
 
 cudaError_t launch_rotate_quant(RQMode mode, const RQArgs& a, cudaStream_t s, bool pdl) {
   const size_t smem = rotate_quant_smem(a.K, a.chunk);
