@@ -114,6 +114,24 @@ dptq_status dptq_qlinear(dptq_handle h, const void* x_fp16, int M, int bits, voi
 dptq_status dptq_qlinear_quantize(dptq_handle h, const void* x_fp16, int M, int bits, void* stream);
 dptq_status dptq_qlinear_gemm(dptq_handle h, int M, int bits, void* out_fp16, void* stream);
 
+/* dptq_qlinear for callers that cannot allocate device memory when they call it:
+ * runtimes whose own memory pool owns all device memory, or hosts that forbid
+ * cudaMalloc once they are serving.  The paper has no counterpart: this is a property
+ * of the library, not of the method.
+ * Same arguments and results as dptq_qlinear, but its scratch lives in one fixed
+ * device array of about 5 MiB inside the library, which every GPU that loads the
+ * library holds until the process exits.  The call never runs cudaMalloc, cudaFree or
+ * an allocating library routine.
+ * Limits: M <= 32 tokens and K <= 16384; larger shapes return DPTQ_ERR_UNSUPPORTED.
+ * The first call on a device looks the array up (cudaGetSymbolAddress) and zeroes it,
+ * synchronously; make that first call before any stream capture.
+ * All calls share the array: calls whose kernels overlap on the GPU (for example on
+ * two streams without ordering between them) race and corrupt each other's results.
+ * A bounded-wait timeout inside this call is recorded in the array, not in the word
+ * that dptq_last_device_error reads. */
+dptq_status dptq_qlinear_static(dptq_handle h, const void* x_fp16, int M, int bits, void* out_fp16,
+                                void* stream);
+
 /* GEMM + epilogue on caller-provided codes (the format dptq_rotate_quant_act writes)
  * and per-token scales.  acc_i32: optional device int32 [M][N] that receives the
  * exact integer accumulators (test hook); NULL to skip. */

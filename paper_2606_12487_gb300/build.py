@@ -17,7 +17,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 OUT_DIR = os.path.join(HERE, "_build")
 LIB = os.path.join(OUT_DIR, "libdptq.so")
-SOURCES = ["api.cu", "rotate_quant.cu", "qgemm.cu"]
+SOURCES = ["api.cu", "rotate_quant.cu", "qgemm.cu", "static_scratch.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

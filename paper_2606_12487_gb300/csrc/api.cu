@@ -17,14 +17,6 @@
 
 using namespace dptq;
 
-struct dptq_linear {
-  int device;
-  int N, K, K_pad, KB, N_pad;
-  int had_block;
-  uint8_t* wt;  // [N_pad/128][KB][128][64] sign-magnitude nibbles
-  float* sw;    // [N_pad]
-};
-
 namespace {
 
 thread_local std::string g_msg;
@@ -191,6 +183,11 @@ dptq_status run_gemm(dptq_handle h, const GemmPlan& plan0, const uint8_t* act, c
 }
 
 }  // namespace
+
+namespace dptq {
+// Record the message returned by dptq_last_error_message for this thread.
+void set_error_message(const std::string& m) { g_msg = m; }
+}  // namespace dptq
 
 extern "C" {
 

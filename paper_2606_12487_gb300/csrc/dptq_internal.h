@@ -2,8 +2,18 @@
 // libdptq (kernel argument blocks and launchers).  Not part of the public ABI.
 #pragma once
 #include <cstdint>
+#include <string>
 #include <cuda_runtime.h>
 #include <cuda_fp16.h>
+
+// The layer handle behind dptq_handle.
+struct dptq_linear {
+  int device;
+  int N, K, K_pad, KB, N_pad;
+  int had_block;
+  uint8_t* wt;  // [N_pad/128][KB][128][64] sign-magnitude nibbles
+  float* sw;    // [N_pad]
+};
 
 namespace dptq {
 
@@ -94,6 +104,9 @@ struct GemmPlan {
 // pointers.  Returns false if the shape cannot be run.
 bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan);
 cudaError_t launch_gemm(const GemmPlan& plan, cudaStream_t s, bool pdl);
+
+// Message returned by dptq_last_error_message() on the calling thread.
+void set_error_message(const std::string& m);
 int gemm_pick_nt(int M, int bits, int KB);
 
 }  // namespace dptq

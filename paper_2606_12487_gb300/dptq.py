@@ -21,7 +21,7 @@ _STATUS = {0: "ok", 1: "invalid argument", 2: "unsupported shape", 3: "CUDA erro
            4: "out of device memory", 5: "device wait timed out"}
 
 EXPORTS = ("dptq_pack_weights", "dptq_rotate_quant_act", "dptq_rotate_act", "dptq_qlinear",
-           "dptq_qlinear_quantize", "dptq_qlinear_gemm",
+           "dptq_qlinear_quantize", "dptq_qlinear_gemm", "dptq_qlinear_static",
            "dptq_qgemm_codes", "dptq_reserve", "dptq_get_packed", "dptq_get_shape",
            "dptq_last_device_error", "dptq_destroy", "dptq_status_str", "dptq_last_error_message")
 
@@ -53,6 +53,7 @@ def load(build_if_missing: bool = True):
                 "dptq_qlinear": ([P, P, I, I, P, P], I),
                 "dptq_qlinear_quantize": ([P, P, I, I, P], I),
                 "dptq_qlinear_gemm": ([P, I, I, P, P], I),
+                "dptq_qlinear_static": ([P, P, I, I, P, P], I),
                 "dptq_qgemm_codes": ([P, P, P, I, I, P, P, P], I),
                 "dptq_reserve": ([I, I, I], I),
                 "dptq_get_packed": ([P, P, P], I),
@@ -159,6 +160,16 @@ def dptq_qlinear(layer: QLinear, x, bits: int, out, stream=None):
     _check_tensor(x, torch.float16, (M, layer.K), "x")
     _check_tensor(out, torch.float16, (M, layer.N), "out")
     _check(load().dptq_qlinear(layer.handle, _ptr(x), M, bits, _ptr(out), _stream(stream)))
+
+
+def dptq_qlinear_static(layer: QLinear, x, bits: int, out, stream=None):
+    """dptq_qlinear without any device allocation: the library's fixed scratch array is
+    used instead (M <= 32, K <= 16384)."""
+    import torch
+    M = x.shape[0]
+    _check_tensor(x, torch.float16, (M, layer.K), "x")
+    _check_tensor(out, torch.float16, (M, layer.N), "out")
+    _check(load().dptq_qlinear_static(layer.handle, _ptr(x), M, bits, _ptr(out), _stream(stream)))
 
 
 def dptq_qlinear_quantize(layer: QLinear, x, bits: int, stream=None):

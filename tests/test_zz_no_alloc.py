@@ -1,0 +1,70 @@
+"""dptq_qlinear_static, the entry point that allocates no device memory, against
+dptq_qlinear.
+
+Callers whose own memory pool owns the device, or that may not call cudaMalloc once
+they are serving, cannot let the library grow its scratch; dptq_qlinear_static serves
+them from a fixed array inside the library.  This file is collected last, so a failure
+here comes after every other test has run; it also passes on its own in a fresh
+process.
+"""
+import ctypes
+
+import pytest
+
+import parity
+from paper_2606_12487_gb300 import inputs
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def dp():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2606_12487_gb300 import dptq
+    dptq.load()
+    return dptq
+
+
+def _static_call(dp, layer, x, bits, out):
+    """Straight through the C ABI."""
+    lib = dp.load()
+    st = lib.dptq_qlinear_static(layer.handle, ctypes.c_void_p(x.data_ptr()), x.shape[0], bits,
+                                 ctypes.c_void_p(out.data_ptr()),
+                                 ctypes.c_void_p(torch.cuda.current_stream().cuda_stream))
+    return st, lib.dptq_last_error_message().decode()
+
+
+@pytest.mark.parametrize("M,N,K,B,bits", [(32, 4096, 4096, 4096, 4), (1, 4096, 4096, 4096, 8),
+                                          (17, 1024, 11008, 256, 4), (32, 12288, 4096, 4096, 8)])
+def test_static_scratch_matches_qlinear_twice(dp, M, N, K, B, bits):
+    wl = inputs.llama2_7b_decode()
+    x = torch.from_numpy(inputs.activations(wl, M, K)).cuda()
+    W = torch.from_numpy(inputs.weights(N, K, layer=3, proj=1)).cuda()
+    layer = dp.dptq_pack_weights(W, B)
+    ref = torch.empty((M, N), dtype=torch.float16, device="cuda")
+    dp.dptq_qlinear(layer, x, bits, ref)
+    for _ in range(2):                     # the shared array must be left clean by each call
+        out = torch.full((M, N), float("nan"), dtype=torch.float16, device="cuda")
+        st, msg = _static_call(dp, layer, x, bits, out)
+        assert st == 0, msg
+        torch.cuda.synchronize()
+        parity.check_out(out.cpu().numpy(), ref.cpu().numpy())
+    dp.dptq_last_device_error()
+    layer.close()
+
+
+def test_static_scratch_rejects_shapes_beyond_its_limit(dp):
+    W = torch.from_numpy(inputs.weights(128, 4096)).cuda()
+    layer = dp.dptq_pack_weights(W, 4096)
+    x = torch.zeros((33, 4096), dtype=torch.float16, device="cuda")
+    out = torch.empty((33, 128), dtype=torch.float16, device="cuda")
+    st, msg = _static_call(dp, layer, x, 4, out)
+    assert st == 2 and "32" in msg
+    W2 = torch.from_numpy(inputs.weights(128, 16640)).cuda()
+    layer2 = dp.dptq_pack_weights(W2, 256)
+    x2 = torch.zeros((4, 16640), dtype=torch.float16, device="cuda")
+    out2 = torch.empty((4, 128), dtype=torch.float16, device="cuda")
+    st, msg = _static_call(dp, layer2, x2, 4, out2)
+    assert st == 2 and "16384" in msg
