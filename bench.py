@@ -207,10 +207,29 @@ class Stack:
 gemm_events_done = []
 
 
+def traffic_record():
+    """DRAM bytes / algorithmic bytes of the GEMM from the committed ncu summary, if the
+    summary was taken on the current kernel source (else None)."""
+    import glob
+    import hashlib
+    src = os.path.join(ROOT, "paper_2606_12487_gb300", "csrc", "qgemm.cu")
+    try:
+        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    except OSError:
+        return None
+    for path in sorted(glob.glob(os.path.join(ROOT, "profiles", "*.md"))):
+        for ln in open(path):
+            if ln.startswith("traffic_record:") and f"sha256/16={sha}" in ln:
+                kv = dict(p.split("=", 1) for p in ln.split() if "=" in p)
+                return int(kv["dram_bytes"]) / int(kv["algorithmic_bytes"]), os.path.basename(path)
+    return None
+
+
 def time_graph(g, stream, steps, warmup, world, device_index, sample_clocks=True):
     import torch
-    for _ in range(warmup):
-        g.replay()
+    with torch.cuda.stream(stream):
+        for _ in range(warmup):
+            g.replay()
     torch.cuda.synchronize()
     barrier(world)
     torch.cuda.synchronize()
@@ -232,8 +251,20 @@ def time_graph(g, stream, steps, warmup, world, device_index, sample_clocks=True
     return ms, (sampler.summary() if sampler else None)
 
 
-def capture(stack, stream):
+class EagerStep:
+    """Stands in for a captured graph: replay() launches the step's kernels directly."""
+
+    def __init__(self, stack, stream):
+        self.stack, self.stream = stack, stream
+
+    def replay(self):
+        self.stack.run(self.stream)
+
+
+def capture(stack, stream, eager=False):
     import torch
+    if eager:
+        return EagerStep(stack, stream)
     g = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g, stream=stream):
         stack.run(stream)
@@ -407,6 +438,8 @@ def main(argv=None):
     ap.add_argument("--m", type=int, default=DEFAULT_M, help="tokens per step (decode batch)")
     ap.add_argument("--sweep", default="1,8", help="extra token counts measured for the m_sweep entry")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--eager", action="store_true",
+                    help="launch the step's kernels directly instead of replaying a CUDA graph")
     ap.add_argument("--layers", type=int, default=0,
                     help="run only the first L layers (small cases for profiler captures; 0 = all)")
     args = ap.parse_args(argv)
@@ -433,7 +466,7 @@ def main(argv=None):
     stream = torch.cuda.Stream(device=device)
 
     stack = Stack(dptq, wl, layers, args.m, device)
-    g = capture(stack, stream)
+    g = capture(stack, stream, args.eager)
     ms, clocks = time_graph(g, stream, args.steps, args.warmup, world, local)
     ms_max = max_over_ranks(ms, world, device)
     value = aggregate_value(args.m, world, ms_max / 1e3)
@@ -447,13 +480,15 @@ def main(argv=None):
         pass
     hbm_peak = float(peaks.get("hbm_gbs", 6800.0))
     achieved = tb / tt / 1e9
+    rec = traffic_record()
+    traffic = rec[0] * tb / n_gemm if rec else None
     e2e_dev_s, e2e_wall_s = e2e_measure(stack, g, stream, max(10, args.steps // 4), world)
     e2e_s = max_over_ranks(e2e_dev_s, world, device)
 
     sweep = {}
     for m in [int(v) for v in args.sweep.split(",") if v]:
         st = Stack(dptq, wl, layers, m, device)
-        gm = capture(st, stream)
+        gm = capture(st, stream, args.eager)
         ms_m, _ = time_graph(gm, stream, max(20, args.steps // 2), args.warmup, world, local, sample_clocks=False)
         ms_m = max_over_ranks(ms_m, world, device)
         tbm, _, ttm, _ = measure_gemm_kernels(st, stream)
@@ -476,7 +511,10 @@ def main(argv=None):
                    "parallelism": f"replicas x{world}", "l2": "weights 3.24 GB > L2 (streamed every step)",
                    "weight_bytes_per_step": weight_bytes},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
-                     "frac": achieved / hbm_peak, "traffic": None, "kernel": "qgemm_kernel",
+                     "frac": achieved / hbm_peak, "traffic": traffic, "kernel": "qgemm_kernel",
+                     "traffic_note": (f"bytes per average launch: ncu DRAM/algorithmic ratio {rec[0]:.3f} "
+                                      f"({rec[1]}) x {tb / n_gemm:.0f} algorithmic bytes") if rec else
+                                     "no capture of the current kernel source",
                      "peak_source": "MEASURED_PEAKS.json hbm_gbs (copy, burst)",
                      "launches_per_step": n_gemm},
         "gemm_tops": to / tt / 1e12,

@@ -4,6 +4,7 @@
 #include <cmath>
 #include <cstdint>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <map>
 #include <mutex>
@@ -185,6 +186,14 @@ dptq_status run_gemm(dptq_handle h, const GemmPlan& plan0, const uint8_t* act, c
 }  // namespace
 
 namespace dptq {
+bool pdl_allowed() {
+  static const bool on = [] {
+    const char* v = std::getenv("DPTQ_PDL");
+    return !(v && v[0] == '0');
+  }();
+  return on;
+}
+
 // Record the message returned by dptq_last_error_message for this thread.
 void set_error_message(const std::string& m) { g_msg = m; }
 }  // namespace dptq

@@ -105,6 +105,10 @@ struct GemmPlan {
 bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan);
 cudaError_t launch_gemm(const GemmPlan& plan, cudaStream_t s, bool pdl);
 
+// Programmatic dependent launch is on unless the environment sets DPTQ_PDL=0 (kernels
+// then start only after their predecessor has finished, e.g. for profilers).
+bool pdl_allowed();
+
 // Message returned by dptq_last_error_message() on the calling thread.
 void set_error_message(const std::string& m);
 int gemm_pick_nt(int M, int bits, int KB);

@@ -561,7 +561,7 @@ static cudaError_t launch_nt(const GemmPlan& plan, cudaStream_t s, bool pdl) {
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = pdl ? 1 : 0;
+  cfg.numAttrs = (pdl && pdl_allowed()) ? 1 : 0;
   return cudaLaunchKernelEx(&cfg, qgemm_kernel<NT, KPS>, plan.args);
 }
 

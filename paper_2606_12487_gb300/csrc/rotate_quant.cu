@@ -334,7 +334,7 @@ cudaError_t launch_rotate_quant(RQMode mode, const RQArgs& a, cudaStream_t s, bo
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = pdl ? 1 : 0;
+  cfg.numAttrs = (pdl && pdl_allowed()) ? 1 : 0;
   cudaError_t e = cudaSuccess;
   switch (mode) {
     case kRQPublic:
