@@ -17,6 +17,11 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 OUT_DIR = os.path.join(HERE, "_build")
 LIB = os.path.join(OUT_DIR, "libdptq.so")
+# DPTQ_TRACE=1 builds a separate library whose kernels record %globaltimer stamps.
+TRACE = os.environ.get("DPTQ_TRACE") == "1"
+if TRACE:
+    OUT_DIR = os.path.join(HERE, "_build_trace")
+    LIB = os.path.join(OUT_DIR, "libdptq.so")
 SOURCES = ["api.cu", "rotate_quant.cu", "qgemm.cu", "static_scratch.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
@@ -30,6 +35,7 @@ def nvcc() -> str:
 
 def _flags():
     return ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I", os.path.join(ROOT, "include"),
+                   *(["-DDPTQ_TRACE"] if TRACE else []),
                    "--ptxas-options=-v" if os.environ.get("DPTQ_PTXAS_V") else "-Xptxas=-O3"]
 
 

@@ -410,8 +410,8 @@ dptq_status dptq_get_packed(dptq_handle h, void* wq_host, float* sw_host) {
       for (int d = 0; d < 2; ++d) {
         const int kk = k + d;
         const int e = kk & 15;  // position in the 16-weight chunk
-        const size_t chunk = (((size_t)(n >> 7) * h->KB + (kk >> 7)) * kWTileBytes) + (n & 127) * 64 +
-                             ((kk & 127) >> 4) * 8;
+        const size_t chunk = (((size_t)(n >> 7) * h->KB + (kk >> 7)) * kWTileBytes) + ((kk & 127) >> 5) * 2048 +
+                             (n & 127) * 16 + (((kk & 127) >> 4) & 1) * 8;
         const int word = e >> 3, i = e & 3, high = (e & 7) >= 4;
         const uint8_t byte = t[chunk + word * 4 + i];
         const int nib = high ? (byte >> 4) & 0xF : byte & 0xF;

@@ -8,6 +8,37 @@
 
 namespace dptq {
 
+// ------------------------------------------------------------------ tracing
+// Built with -DDPTQ_TRACE (a separate library, see build.py), kernels record
+// %globaltimer stamps per CTA at fixed slots of a 128-entry row of the buffer set by
+// dptq_trace_set(); otherwise the trace points compile to nothing.
+#ifdef DPTQ_TRACE
+// One copy per translation unit; dptq_trace_set() sets the GEMM's.
+static __device__ unsigned long long* g_dptq_trace = nullptr;
+__device__ __forceinline__ unsigned long long trace_now() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+#define DPTQ_TRACE_POINT(buf, slot) \
+  do {                              \
+    if (buf) (buf)[blockIdx.x * 128 + (slot)] = ::dptq::trace_now(); \
+  } while (0)
+#define DPTQ_TRACE_VALUE(buf, slot, v) \
+  do {                                 \
+    if (buf) (buf)[blockIdx.x * 128 + (slot)] = (unsigned long long)(v); \
+  } while (0)
+#define DPTQ_TRACE_BUF() ::dptq::g_dptq_trace
+#else
+#define DPTQ_TRACE_POINT(buf, slot) \
+  do {                              \
+  } while (0)
+#define DPTQ_TRACE_VALUE(buf, slot, v) \
+  do {                                 \
+  } while (0)
+#define DPTQ_TRACE_BUF() nullptr
+#endif
+
 // Device error codes written to the library's error word (host maps them to status).
 enum DeviceError : int {
   kDevOk = 0,
@@ -128,6 +159,17 @@ __device__ __forceinline__ void mma_f8(uint32_t d_tmem, uint64_t adesc, uint64_t
       "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
+// D[tmem] (+)= A[tmem] * B[smem]^T: A read from tensor memory (one row per lane, four
+// FP8 K-elements per 32-bit column, lowest K in the lowest byte).
+__device__ __forceinline__ void mma_f8_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint32_t idesc,
+                                          uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], [%1], %2, %3, p;\n\t}\n" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
 // Arrive once on `bar` when every MMA issued so far by this thread has completed.
 __device__ __forceinline__ void mma_commit(uint64_t* bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
@@ -162,6 +204,21 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
         "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]),
         "=r"(r[15])
       : "r"(taddr));
+}
+// 32 TMEM lanes (one per thread) x 32 consecutive 32-bit columns, from registers.
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
+      "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+      "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]),
+      "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(r[16]),
+      "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]),
+      "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
+      : "memory");
+}
+__device__ __forceinline__ void tmem_st_wait() {
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
 __device__ __forceinline__ void tmem_ld_wait() {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");

@@ -11,7 +11,7 @@ struct dptq_linear {
   int device;
   int N, K, K_pad, KB, N_pad;
   int had_block;
-  uint8_t* wt;  // [N_pad/128][KB][128][64] sign-magnitude nibbles
+  uint8_t* wt;  // [N_pad/128][KB][4 chunks of 32 k][128 rows][16 B] sign-magnitude nibbles
   float* sw;    // [N_pad]
 };
 
@@ -69,7 +69,7 @@ cudaError_t launch_codes_to_act(const CodesArgs& a, cudaStream_t s);
 
 // ------------------------------------------------------------------ GEMM
 struct GemmArgs {
-  const uint8_t* wt;   // [NTw][KB][128][64] packed sign-magnitude nibbles
+  const uint8_t* wt;   // [NTw][KB][4][128][16] packed sign-magnitude nibbles (chunk-major tiles)
   const uint8_t* act;  // [planes][KB][M_pad][128] E4M3, rows pre-swizzled
   const float* sa;     // [>= M] per-token scales
   const float* sw;     // [>= N] per-channel scales
@@ -85,7 +85,9 @@ struct GemmArgs {
   int seg_iters;       // iterations per exact fp32 accumulation segment
   int segs;            // accumulator segments per tile
   int nbuf;            // TMEM accumulator buffers (1 or 2)
-  int stages;          // shared-memory pipeline depth
+  int stages;          // bulk-copy ring depth
+  int conv_slots;      // widened-weight ring depth
+  uint32_t a_col0;     // first TMEM column of the widened-weight slots (A operand in TMEM)
   int dp_tiles;        // tiles processed whole, round-robin, before the stream-K part
   long long sk_iters;  // stream-K iterations (tiles after dp_tiles, times KI)
   uint32_t tmem_cols;

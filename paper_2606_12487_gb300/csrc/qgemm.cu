@@ -46,6 +46,7 @@ constexpr int kGemmThreads = 32 * (kEpiWarp0 + kNumEpiWarps);   // 448
 constexpr int kConvThreads = 32 * kNumConvWarps;
 constexpr int kConvBytes = 128 * 128;   // one weight tile widened to E4M3
 constexpr int kMaxStages = 8;
+constexpr int kMaxConvSlots = 4;
 constexpr int kSmemLimit = 232448;      // 227 KB opt-in dynamic shared memory per CTA
 constexpr int kBarrierBytes = 1024;
 
@@ -125,37 +126,46 @@ __device__ __forceinline__ uint32_t widen_hi(uint32_t w) {
   return ((w >> 4) & 0x07070707u) | (w & 0x80808080u);
 }
 
-// Shared-memory layout of one pipeline stage: KPS widened weight tiles (1024-aligned
-// swizzle atoms), KPS x planes token tiles, then the KPS packed weight tiles.
+// Shared-memory layout: a ring of `conv_slots` widened weight slots (KPS tiles of 16 KB
+// each, 1024-aligned swizzle atoms; absent when the widened weights live in tensor
+// memory) followed by the `stages`-deep ring of bulk-copy slots.  A bulk-copy slot holds
+// KPS x planes token tiles and the KPS packed weight tiles of one stage.
 template <int NT, int KPS>
 struct Smem {
   static constexpr int kActBytes = NT * 128;  // one plane of one token tile
   uint8_t* base;
   int planes;
-  int stage_bytes;
-  __device__ __forceinline__ Smem(uint8_t* b, int p) : base(b), planes(p) {
-    stage_bytes = KPS * (kConvBytes + p * kActBytes + kWTileBytes);
+  int conv_slots;
+  int slot_bytes;
+  __device__ __forceinline__ Smem(uint8_t* b, int p, int cs) : base(b), planes(p), conv_slots(cs) {
+    slot_bytes = KPS * (p * kActBytes + kWTileBytes);
   }
-  __device__ __forceinline__ uint8_t* conv(int s, int h) const { return base + s * stage_bytes + h * kConvBytes; }
-  __device__ __forceinline__ uint8_t* act(int s, int h, int p) const {
-    return base + s * stage_bytes + KPS * kConvBytes + (h * planes + p) * kActBytes;
+  __device__ __forceinline__ uint8_t* conv(int c, int h) const { return base + (c * KPS + h) * kConvBytes; }
+  __device__ __forceinline__ uint8_t* slot(int s) const {
+    return base + conv_slots * KPS * kConvBytes + s * slot_bytes;
   }
-  __device__ __forceinline__ uint8_t* wpack(int s) const {
-    return base + s * stage_bytes + KPS * (kConvBytes + planes * kActBytes);
-  }
+  __device__ __forceinline__ uint8_t* act(int s, int h, int p) const { return slot(s) + (h * planes + p) * kActBytes; }
+  __device__ __forceinline__ uint8_t* wpack(int s) const { return slot(s) + KPS * planes * kActBytes; }
+  __device__ __forceinline__ uint8_t* end(int S) const { return slot(S); }
 };
 
 template <int NT, int KPS>
 __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a) {
+  // Two-block stages (token tiles of up to 64, weight streaming) widen the weights
+  // straight into tensor memory and feed the MMA's A operand from there; one-block
+  // stages widen into shared memory.
+  constexpr bool kATmem = (KPS == 2);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int S = a.stages;
-  const Smem<NT, KPS> sm(smem, a.planes);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + S * sm.stage_bytes);
-  uint64_t* full = bars;
-  uint64_t* convb = bars + kMaxStages;
-  uint64_t* empty = bars + 2 * kMaxStages;
-  uint64_t* tfull = bars + 3 * kMaxStages;
+  const int CS = a.conv_slots;
+  const Smem<NT, KPS> sm(smem, a.planes, kATmem ? 0 : CS);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sm.end(S));
+  uint64_t* full = bars;                     // slot s: copies landed
+  uint64_t* empty = bars + kMaxStages;       // slot s: MMA done with it
+  uint64_t* cfull = bars + 2 * kMaxStages;   // widened slot c: written
+  uint64_t* cempty = cfull + kMaxConvSlots;  // widened slot c: MMA done with it
+  uint64_t* tfull = cempty + kMaxConvSlots;
   uint64_t* tempty = tfull + 2;
   uint64_t* drain = tempty + 2;
   uint64_t* esync = drain + 1;   // epilogue-group barrier (4 warps), bounded waits
@@ -166,12 +176,17 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  unsigned long long* const tr = DPTQ_TRACE_BUF();
+  if (threadIdx.x == 0) DPTQ_TRACE_POINT(tr, 0);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&convb[s], kNumConvWarps);
       mbar_init(&empty[s], 1);
+    }
+    for (int c = 0; c < CS; ++c) {
+      mbar_init(&cfull[c], kNumConvWarps);
+      mbar_init(&cempty[c], 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&tfull[b], 1);
@@ -191,6 +206,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_base_sh;
+  if (threadIdx.x == 0) DPTQ_TRACE_POINT(tr, 1);
   pdl_launch_dependents();
 
   UnitIter iter;
@@ -222,6 +238,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
         for (int it = un.i0; it < un.i1; ++it, ++g, rg.next(), wsrc += w_bytes, asrc += KPS * kb_stride) {
           const int s = rg.s;
           if (!mbar_wait(&empty[s], rg.ph ^ 1u, abort_flag, a.err, kDevTimeoutEmpty)) goto producer_done;
+          if (g < 16) DPTQ_TRACE_POINT(tr, 8 + g);
           mbar_arrive_expect_tx(&full[s], tx);
           bulk_g2s(sm.wpack(s), wsrc, w_bytes, &full[s], pol_w);
           if (waited) {
@@ -229,7 +246,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
             for (int h = 0; h < KPS; ++h)
               for (int p = 0; p < a.planes; ++p)
                 bulk_g2s(sm.act(s, h, p), asrc + h * kb_stride + p * plane_stride, act_bytes, &full[s], pol_a);
+            if (g < 16) DPTQ_TRACE_POINT(tr, 24 + g);
           } else {
+            if (g < 16) DPTQ_TRACE_POINT(tr, 24 + g);
             pend_src[npend++] = asrc;   // stage index of pending entry i is i
             if (npend == S) {
               pdl_wait();
@@ -262,40 +281,71 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
+      // One thread issues every MMA, so the loop body is kept short: descriptors and
+      // TMEM addresses advance by additions, segment boundaries by a countdown.
       const uint32_t idesc = idesc_e4m3_m128(NT);
-      Ring rg(S);
-      int u = 0;
+      const int planes = a.planes;
+      // Shared-memory descriptors hold address >> 4 in their low bits, so a byte offset
+      // `o` into a region is `desc + (o >> 4)`.
+      const uint64_t act_desc0 = sdesc_sw128(smem_u32(sm.act(0, 0, 0)));
+      const uint64_t conv_desc0 = kATmem ? 0 : sdesc_sw128(smem_u32(sm.conv(0, 0)));
+      const uint32_t slot_step = (uint32_t)(sm.slot_bytes >> 4);
+      const uint32_t act_step = (uint32_t)(Smem<NT, KPS>::kActBytes >> 4);
+      const uint32_t a_tmem0 = tmem_base + a.a_col0;
+      Ring rg(S), rc(CS);
+      int u = 0, mma_done = 0;
       while (iter.next(un)) {
         const int b = a.nbuf == 2 ? (u & 1) : 0;
         const uint32_t tpar = ((a.nbuf == 2 ? (u >> 1) : u) & 1) ^ 1;
         if (!mbar_wait(&tempty[b], tpar, abort_flag, a.err, kDevTimeoutTmemEmpty)) break;
         tc_fence_after();
-        const uint32_t dbase = tmem_base + (uint32_t)(b * NT * a.segs);
-        const int seg0 = un.i0 / a.seg_iters;
+        uint32_t d = tmem_base + (uint32_t)(b * NT * a.segs);
+        int seg_left = a.seg_iters - un.i0 % a.seg_iters;   // iterations left in this segment
+        uint32_t fresh = 1;
         bool ok = true;
-        for (int it = un.i0; it < un.i1; ++it, rg.next()) {
-          const int s = rg.s;
-          if (!mbar_wait(&convb[s], rg.ph, abort_flag, a.err, kDevTimeoutConv)) {
+        for (int it = un.i0; it < un.i1; ++it, rg.next(), rc.next()) {
+          const int s = rg.s, c = rc.s;
+          if (!mbar_wait(&cfull[c], rc.ph, abort_flag, a.err, kDevTimeoutConv)) {
             ok = false;
             break;
           }
+          const int gm = it - un.i0 + mma_done;
+          if (gm < 16) DPTQ_TRACE_POINT(tr, 72 + gm);
           tc_fence_after();
-          const uint32_t d = dbase + (uint32_t)((it / a.seg_iters - seg0) * NT);
-          const bool fresh = (it == un.i0) || (it % a.seg_iters == 0);
+          if (seg_left == 0) {   // next exact-accumulation segment: next accumulator
+            d += NT;
+            fresh = 1;
+            seg_left = a.seg_iters;
+          }
+          const uint64_t bd_slot = act_desc0 + (uint64_t)(s * slot_step);
 #pragma unroll
           for (int h = 0; h < KPS; ++h) {
-            const uint64_t ad = sdesc_sw128(smem_u32(sm.conv(s, h)));
-            for (int p = 0; p < a.planes; ++p) {
-              const uint64_t bd = sdesc_sw128(smem_u32(sm.act(s, h, p)));
+            const uint64_t ad = conv_desc0 + (uint64_t)((c * KPS + h) * (kConvBytes >> 4));
+            const uint32_t at = a_tmem0 + (uint32_t)((c * KPS + h) * 32);   // 32 columns per k-block
 #pragma unroll
-              for (int ks = 0; ks < 4; ++ks)   // 4 x (K = 32 FP8 elements = 32 bytes)
-                mma_f8(d, ad + 2 * ks, bd + 2 * ks, idesc, (fresh && h == 0 && p == 0 && ks == 0) ? 0u : 1u);
+            for (int p = 0; p < 2; ++p) {
+              if (p < planes) {
+                const uint64_t bd = bd_slot + (uint64_t)((h * planes + p) * act_step);
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks) {   // 4 x (K = 32 FP8 elements = 32 bytes = 8 columns)
+                  const uint32_t accumulate = (h | p | ks) ? 1u : (fresh ^ 1u);
+                  if (kATmem)
+                    mma_f8_ts(d, at + (uint32_t)(8 * ks), bd + 2 * ks, idesc, accumulate);
+                  else
+                    mma_f8(d, ad + 2 * ks, bd + 2 * ks, idesc, accumulate);
+                }
+              }
             }
           }
           mma_commit(&empty[s]);
+          mma_commit(&cempty[c]);
+          if (gm < 16) DPTQ_TRACE_POINT(tr, 88 + gm);
+          fresh = 0;
+          --seg_left;
         }
         if (!ok) break;
         mma_commit(&tfull[b]);
+        mma_done += un.i1 - un.i0;
         ++u;
       }
       // Every MMA this thread issued must be complete before TMEM is released.
@@ -306,40 +356,76 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
   } else if (warp < kEpiWarp0) {
     // ------------------------------------------------------------ converters
     const int ctid = threadIdx.x - kConvWarp0 * 32;   // 0..255
-    Ring rg(S);
+    Ring rg(S), rc(CS);
+    int cvt_done = 0;
     while (iter.next(un)) {
       bool ok = true;
-      for (int it = un.i0; it < un.i1; ++it, rg.next()) {
-        const int s = rg.s;
-        if (!mbar_wait(&full[s], rg.ph, abort_flag, a.err, kDevTimeoutFull)) {
+      for (int it = un.i0; it < un.i1; ++it, rg.next(), rc.next()) {
+        const int s = rg.s, c = rc.s;
+        if (!mbar_wait(&full[s], rg.ph, abort_flag, a.err, kDevTimeoutFull) ||
+            !mbar_wait(&cempty[c], rc.ph ^ 1u, abort_flag, a.err, kDevTimeoutConv)) {
           ok = false;
           break;
         }
+        const int gc = it - un.i0 + cvt_done;
+        if (ctid == 0 && gc < 16) DPTQ_TRACE_POINT(tr, 40 + gc);
         const uint8_t* __restrict__ wp = sm.wpack(s);
-        // Each thread widens 2 * KPS x 16 packed bytes: (tile h, row r, chunks j0 and
-        // j0 + 1) of 16 weights each.  All loads are issued before any store.
-        uint4 w[2 * KPS];
+        if constexpr (kATmem) {
+          // Warp (lane quarter q, half hs) widens k-block hs of rows 32q..32q+31: each
+          // thread reads its row's 64 packed bytes (4 chunks of 32 k) and stores 32 columns
+          // of its TMEM lane.
+          tc_fence_after();
+          const int q = warp & 3;
+          const int hs = (warp - kConvWarp0) >> 2;
+          const uint8_t* src = wp + hs * kWTileBytes + (q * 32 + lane) * 16;
+          uint4 w[4];
 #pragma unroll
-        for (int i = 0; i < 2 * KPS; ++i) {
-          const int p = i * kConvThreads + ctid;   // 16-byte unit: tile p >> 9
-          w[i] = *reinterpret_cast<const uint4*>(wp + (p >> 9) * kWTileBytes + ((p & 511) >> 2) * 64 + (p & 3) * 16);
-        }
+          for (int j = 0; j < 4; ++j) w[j] = *reinterpret_cast<const uint4*>(src + j * 2048);
+          uint32_t v[32];
 #pragma unroll
-        for (int i = 0; i < 2 * KPS; ++i) {
-          const int p = i * kConvThreads + ctid;
-          const int q = p & 511;
-          const int r = q >> 2, j0 = (q & 3) * 2;
-          uint8_t* row = sm.conv(s, p >> 9) + r * 128;
-          *reinterpret_cast<uint4*>(row + ((j0 ^ (r & 7)) << 4)) =
-              make_uint4(widen_lo(w[i].x), widen_hi(w[i].x), widen_lo(w[i].y), widen_hi(w[i].y));
-          *reinterpret_cast<uint4*>(row + (((j0 + 1) ^ (r & 7)) << 4)) =
-              make_uint4(widen_lo(w[i].z), widen_hi(w[i].z), widen_lo(w[i].w), widen_hi(w[i].w));
+          for (int j = 0; j < 4; ++j) {
+            v[8 * j + 0] = widen_lo(w[j].x);
+            v[8 * j + 1] = widen_hi(w[j].x);
+            v[8 * j + 2] = widen_lo(w[j].y);
+            v[8 * j + 3] = widen_hi(w[j].y);
+            v[8 * j + 4] = widen_lo(w[j].z);
+            v[8 * j + 5] = widen_hi(w[j].z);
+            v[8 * j + 6] = widen_lo(w[j].w);
+            v[8 * j + 7] = widen_hi(w[j].w);
+          }
+          tmem_st32(tmem_base + ((uint32_t)(q * 32) << 16) + a.a_col0 + (uint32_t)((c * KPS + hs) * 32), v);
+          tmem_st_wait();
+          tc_fence_before();
+        } else {
+          // Each thread widens 2 * KPS x 16 packed bytes: (tile h, row r, 16-byte chunk jj
+          // = 32 weights) into swizzled chunks 2jj and 2jj + 1 of row r.  All loads are
+          // issued before any store.
+          uint4 w[2 * KPS];
+#pragma unroll
+          for (int i = 0; i < 2 * KPS; ++i) {
+            const int p = i * kConvThreads + ctid;   // 16-byte unit: tile p >> 9
+            const int qq = p & 511;
+            w[i] = *reinterpret_cast<const uint4*>(wp + (p >> 9) * kWTileBytes + (qq & 3) * 2048 + (qq >> 2) * 16);
+          }
+#pragma unroll
+          for (int i = 0; i < 2 * KPS; ++i) {
+            const int p = i * kConvThreads + ctid;
+            const int qq = p & 511;
+            const int r = qq >> 2, j0 = (qq & 3) * 2;
+            uint8_t* row = sm.conv(c, p >> 9) + r * 128;
+            *reinterpret_cast<uint4*>(row + ((j0 ^ (r & 7)) << 4)) =
+                make_uint4(widen_lo(w[i].x), widen_hi(w[i].x), widen_lo(w[i].y), widen_hi(w[i].y));
+            *reinterpret_cast<uint4*>(row + (((j0 + 1) ^ (r & 7)) << 4)) =
+                make_uint4(widen_lo(w[i].z), widen_hi(w[i].z), widen_lo(w[i].w), widen_hi(w[i].w));
+          }
+          fence_proxy_async_smem();
         }
-        fence_proxy_async_smem();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&convb[s]);
+        if (lane == 0) mbar_arrive(&cfull[c]);
+        if (ctid == 0 && gc < 16) DPTQ_TRACE_POINT(tr, 56 + gc);
       }
       if (!ok) break;
+      cvt_done += un.i1 - un.i0;
     }
   } else {
     // ------------------------------------------------------------ epilogue
@@ -367,6 +453,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
       const int b = a.nbuf == 2 ? (u & 1) : 0;
       const uint32_t tpar = (a.nbuf == 2 ? (u >> 1) : u) & 1;
       if (!mbar_wait(&tfull[b], tpar, abort_flag, a.err, kDevTimeoutTmemFull)) break;
+      if (etid == 0 && u < 4) DPTQ_TRACE_POINT(tr, 104 + u);
       tc_fence_after();
       const int nt = un.tile / a.m_tiles;
       const int mt = un.tile - nt * a.m_tiles;
@@ -408,6 +495,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
           for (int i = 0; i < 16; ++i) atomicAdd(wsl + (c0 + i) * 128 + q * 32 + lane, acc[i]);
         }
       }
+      if (etid == 0 && u < 4) DPTQ_TRACE_POINT(tr, 112 + u);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&tempty[b]);
@@ -450,7 +538,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
         }
         if (!epi_sync()) break;
       }
+      if (etid == 0 && u <= 4) DPTQ_TRACE_POINT(tr, 108 + u - 1);
     }
+    if (etid == 0) DPTQ_TRACE_VALUE(tr, 122, u);
   }
 
   tc_fence_before();
@@ -459,6 +549,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
     tc_fence_after();
     tmem_dealloc(tmem_base, a.tmem_cols);
   }
+  if (threadIdx.x == 0) DPTQ_TRACE_POINT(tr, 120);
 }
 
 // ------------------------------------------------------------------ host planning
@@ -476,8 +567,8 @@ int gemm_pick_nt(int M, int bits, int KB) {
 // keep one k-block per stage for a deeper ring.
 static int kps_for(int nt) { return nt <= 64 ? 2 : 1; }
 
-static int smem_for(int nt, int kps, int stages, int planes) {
-  return 1024 + stages * kps * (kConvBytes + planes * nt * 128 + kWTileBytes) + kBarrierBytes;
+static int smem_for(int nt, int kps, int stages, int planes, int conv_slots) {
+  return 1024 + conv_slots * kps * kConvBytes + stages * kps * (planes * nt * 128 + kWTileBytes) + kBarrierBytes;
 }
 
 bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan) {
@@ -506,12 +597,24 @@ bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan) {
     }
   }
   if (nt * segs > 512) return false;
+  // Widened weights live in TMEM for two-block stages (A operand read from TMEM; 4 slots
+  // of 64 columns after the accumulators), else in shared memory: as many slots as fit
+  // next to at least 4 bulk-copy stages (the converters may run that far ahead of MMA
+  // completion).
+  const bool a_tmem = kps == 2;
+  int conv_slots = kMaxConvSlots;
+  if (!a_tmem)
+    while (conv_slots > 2 && smem_for(nt, kps, 4, planes, conv_slots) > kSmemLimit) --conv_slots;
+  const int smem_conv = a_tmem ? 0 : conv_slots;
   int stages = kMaxStages;
-  while (stages > 2 && smem_for(nt, kps, stages, planes) > kSmemLimit) --stages;
-  if (smem_for(nt, kps, stages, planes) > kSmemLimit) return false;
-  const int nbuf = 2 * nt * segs <= 512 ? 2 : 1;
+  while (stages > 2 && smem_for(nt, kps, stages, planes, smem_conv) > kSmemLimit) --stages;
+  if (smem_for(nt, kps, stages, planes, smem_conv) > kSmemLimit) return false;
+  const int a_cols = a_tmem ? conv_slots * kps * 32 : 0;
+  const int nbuf = 2 * nt * segs + a_cols <= 512 ? 2 : 1;
+  if (nbuf * nt * segs + a_cols > 512) return false;
+  const int acc_cols = nbuf * nt * segs;
   uint32_t cols = 32;
-  while (cols < (uint32_t)(nbuf * nt * segs)) cols <<= 1;
+  while (cols < (uint32_t)(acc_cols + a_cols)) cols <<= 1;
 
   const int KI = KB / kps;
   const int M_pad = round_up(M, nt);
@@ -528,7 +631,7 @@ bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan) {
   plan.kps = kps;
   plan.M_pad = M_pad;
   plan.grid = G;
-  plan.smem_bytes = smem_for(nt, kps, stages, planes);
+  plan.smem_bytes = smem_for(nt, kps, stages, planes, smem_conv);
   a.M = M;
   a.N = N;
   a.M_pad = M_pad;
@@ -540,7 +643,9 @@ bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan) {
   a.seg_iters = seg_iters;
   a.segs = segs;
   a.nbuf = nbuf;
+  a.a_col0 = (uint32_t)acc_cols;
   a.stages = stages;
+  a.conv_slots = conv_slots;
   a.dp_tiles = (int)dp;
   a.sk_iters = (tiles - dp) * KI;
   a.tmem_cols = cols;
@@ -585,3 +690,10 @@ cudaError_t launch_gemm(const GemmPlan& plan, cudaStream_t s, bool pdl) {
 }
 
 }  // namespace dptq
+
+#ifdef DPTQ_TRACE
+// Trace builds only: set (or clear with NULL) the device buffer of 128 stamps per CTA.
+extern "C" int dptq_trace_set(void* dev_buffer) {
+  return (int)cudaMemcpyToSymbol(dptq::g_dptq_trace, &dev_buffer, sizeof(dev_buffer));
+}
+#endif

@@ -291,7 +291,8 @@ __global__ void __launch_bounds__(kRQThreads) rotate_quant_kernel(const RQArgs a
     } else if constexpr (MODE == kRQWeights) {
       // 16 weights -> 8 bytes.  Nibble = sign (bit 3) | magnitude (bits 0-2); word 0
       // byte i holds k0+i (low nibble) and k0+4+i (high nibble), word 1 holds k0+8+i
-      // and k0+12+i, so that the GEMM widens a word with two masks per half.
+      // and k0+12+i, so that the GEMM widens a word with two masks per half.  A tile of
+      // 128 rows x 128 k is stored as 4 column chunks of 32 k, each [128 rows][16 B].
       uint8_t* wt = static_cast<uint8_t*>(a.out);
       const int nchunks = a.KB * 8;
       for (int ch = tid; ch < nchunks; ch += kRQThreads) {
@@ -311,7 +312,10 @@ __global__ void __launch_bounds__(kRQThreads) rotate_quant_kernel(const RQArgs a
           w0 |= (nib[i] | (nib[4 + i] << 4)) << (8 * i);
           w1 |= (nib[8 + i] | (nib[12 + i] << 4)) << (8 * i);
         }
-        const size_t off = (((size_t)(row >> 7) * a.KB + kb) * kWTileBytes) + (row & 127) * 64 + j * 8;
+        // tile [16-byte chunk j / 2][row][16 B]: the 32 rows a warp reads side by side
+        // are contiguous
+        const size_t off = (((size_t)(row >> 7) * a.KB + kb) * kWTileBytes) + (j >> 1) * 2048 + (row & 127) * 16 +
+                           (j & 1) * 8;
         *reinterpret_cast<uint2*>(wt + off) = make_uint2(w0, w1);
       }
     }
