@@ -105,6 +105,39 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
   }
 }
 
+// The same wait for a whole, converged warp: every lane polls, the result is the same
+// for all lanes, and lane 0 decides a time-out.  The phase waited on must not be able to
+// advance twice while the warp polls (true for every ring here: its next phase needs an
+// action of this warp first).
+__device__ __forceinline__ bool mbar_wait_warp(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                               int* err, int code) {
+  if (__all_sync(0xffffffffu, mbar_try_wait(bar, parity))) return true;
+  const long long t0 = clock64();
+  while (true) {
+    if (__all_sync(0xffffffffu, mbar_try_wait(bar, parity))) return true;
+    __nanosleep(20);
+    int stop = 0;
+    if ((threadIdx.x & 31) == 0) stop = *abort_flag ? 1 : (clock64() - t0 > kWaitTimeoutCycles ? 2 : 0);
+    stop = __shfl_sync(0xffffffffu, stop, 0);
+    if (stop) {
+      if (stop == 2 && (threadIdx.x & 31) == 0) {
+        *abort_flag = 1;
+        atomicCAS(err, 0, code);
+      }
+      return false;
+    }
+  }
+}
+
+// One lane of a converged warp (the lowest) gets true.  Single-thread tcgen05 and bulk
+// copy issue is much faster from an elected lane of a warp whose control flow is uniform
+// than from a thread that runs its loop alone.
+__device__ __forceinline__ bool elect_one() {
+  uint32_t p = 0;
+  asm volatile("{\n\t.reg .pred P;\n\telect.sync _|P, 0xffffffff;\n\tselp.b32 %0, 1, 0, P;\n\t}\n" : "=r"(p));
+  return p != 0;
+}
+
 // ------------------------------------------------------------------ bulk copies (TMA engine)
 __device__ __forceinline__ uint64_t l2_policy_evict_first() {
   uint64_t pol;

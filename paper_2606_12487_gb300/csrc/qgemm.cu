@@ -215,109 +215,120 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
-    if (lane == 0) {
-      const uint64_t pol_w = l2_policy_evict_first();   // weights are streamed once
-      const uint64_t pol_a = l2_policy_evict_last();    // activations are re-read per n-tile
-      const uint32_t act_bytes = (uint32_t)NT * 128;
-      const uint32_t w_bytes = (uint32_t)KPS * kWTileBytes;
-      const uint32_t tx = w_bytes + (uint32_t)(KPS * a.planes) * act_bytes;
-      const size_t plane_stride = (size_t)a.KB * a.M_pad * 128;
-      const size_t kb_stride = (size_t)a.M_pad * 128;
-      // Weight tiles do not depend on the previous kernel; the first `S` stages are
-      // requested before waiting for it (programmatic dependent launch) and their
-      // activation halves are issued once the previous kernel has finished.
-      bool waited = false;
-      int npend = 0;
-      Ring rg(S);
-      int g = 0;
-      while (iter.next(un)) {
-        const int nt = un.tile / a.m_tiles;
-        const int mt = un.tile - nt * a.m_tiles;
-        const uint8_t* wsrc = a.wt + ((size_t)nt * a.KB + (size_t)un.i0 * KPS) * kWTileBytes;
-        const uint8_t* asrc = a.act + ((size_t)un.i0 * KPS * a.M_pad + (size_t)mt * NT) * 128;
-        for (int it = un.i0; it < un.i1; ++it, ++g, rg.next(), wsrc += w_bytes, asrc += KPS * kb_stride) {
-          const int s = rg.s;
-          if (!mbar_wait(&empty[s], rg.ph ^ 1u, abort_flag, a.err, kDevTimeoutEmpty)) goto producer_done;
+    // Whole warp, uniform control flow; the elected leader issues the copies.
+    const bool leader = elect_one();
+    const uint64_t pol_w = l2_policy_evict_first();   // weights are streamed once
+    const uint64_t pol_a = l2_policy_evict_last();    // activations are re-read per n-tile
+    const uint32_t act_bytes = (uint32_t)NT * 128;
+    const uint32_t w_bytes = (uint32_t)KPS * kWTileBytes;
+    const uint32_t tx = w_bytes + (uint32_t)(KPS * a.planes) * act_bytes;
+    const size_t plane_stride = (size_t)a.KB * a.M_pad * 128;
+    const size_t kb_stride = (size_t)a.M_pad * 128;
+    auto issue_act = [&](int slot, const uint8_t* src) {
+#pragma unroll
+      for (int h = 0; h < KPS; ++h)
+        for (int pl = 0; pl < a.planes; ++pl)
+          bulk_g2s(sm.act(slot, h, pl), src + h * kb_stride + pl * plane_stride, act_bytes, &full[slot], pol_a);
+    };
+    // Weight tiles do not depend on the previous kernel; the first `S` stages are
+    // requested before waiting for it (programmatic dependent launch) and their
+    // activation halves are issued once the previous kernel has finished.
+    bool waited = false;
+    int npend = 0;
+    Ring rg(S);
+    int g = 0;
+    bool ok = true;
+    while (ok && iter.next(un)) {
+      const int nt = un.tile / a.m_tiles;
+      const int mt = un.tile - nt * a.m_tiles;
+      const uint8_t* wsrc = a.wt + ((size_t)nt * a.KB + (size_t)un.i0 * KPS) * kWTileBytes;
+      const uint8_t* asrc = a.act + ((size_t)un.i0 * KPS * a.M_pad + (size_t)mt * NT) * 128;
+      for (int it = un.i0; it < un.i1; ++it, ++g, rg.next(), wsrc += w_bytes, asrc += KPS * kb_stride) {
+        const int s = rg.s;
+        if (!mbar_wait_warp(&empty[s], rg.ph ^ 1u, abort_flag, a.err, kDevTimeoutEmpty)) {
+          ok = false;
+          break;
+        }
+        if (leader) {
           if (g < 16) DPTQ_TRACE_POINT(tr, 8 + g);
           mbar_arrive_expect_tx(&full[s], tx);
           bulk_g2s(sm.wpack(s), wsrc, w_bytes, &full[s], pol_w);
-          if (waited) {
-#pragma unroll
-            for (int h = 0; h < KPS; ++h)
-              for (int p = 0; p < a.planes; ++p)
-                bulk_g2s(sm.act(s, h, p), asrc + h * kb_stride + p * plane_stride, act_bytes, &full[s], pol_a);
-            if (g < 16) DPTQ_TRACE_POINT(tr, 24 + g);
-          } else {
-            if (g < 16) DPTQ_TRACE_POINT(tr, 24 + g);
-            pend_src[npend++] = asrc;   // stage index of pending entry i is i
-            if (npend == S) {
-              pdl_wait();
-              waited = true;
-              for (int i = 0; i < npend; ++i)
-                for (int h = 0; h < KPS; ++h)
-                  for (int p = 0; p < a.planes; ++p)
-                    bulk_g2s(sm.act(i, h, p), pend_src[i] + h * kb_stride + p * plane_stride, act_bytes,
-                             &full[i], pol_a);
-              npend = 0;
-            }
-          }
+          if (waited)
+            issue_act(s, asrc);
+          else
+            pend_src[npend] = asrc;   // stage index of pending entry i is i
+          if (g < 16) DPTQ_TRACE_POINT(tr, 24 + g);
         }
+        if (!waited && ++npend == S) {
+          pdl_wait();
+          waited = true;
+          __syncwarp();
+          if (leader)
+            for (int i = 0; i < npend; ++i) issue_act(i, pend_src[i]);
+          npend = 0;
+        }
+        __syncwarp();
       }
-      if (!waited) {
-        pdl_wait();
-        for (int i = 0; i < npend; ++i)
-          for (int h = 0; h < KPS; ++h)
-            for (int p = 0; p < a.planes; ++p)
-              bulk_g2s(sm.act(i, h, p), pend_src[i] + h * kb_stride + p * plane_stride, act_bytes, &full[i], pol_a);
-      }
-    producer_done:
-      // Do not leave the CTA while copies into its shared memory may be in flight.
-      if (*abort_flag) {
-        volatile int no_abort = 0;
-        for (int gg = (g > S ? g - S : 0); gg < g; ++gg)
-          mbar_wait(&full[gg % S], (gg / S) & 1, &no_abort, a.err, kDevTimeoutDrain);
-      }
+    }
+    // Stages armed before the wait for the previous kernel still expect their
+    // activation bytes (also after an abort, so that the drain below completes).
+    if (!waited) {
+      pdl_wait();
+      __syncwarp();
+      if (leader)
+        for (int i = 0; i < npend; ++i) issue_act(i, pend_src[i]);
+    }
+    __syncwarp();
+    // Do not leave the CTA while copies into its shared memory may be in flight.
+    if (*abort_flag) {
+      volatile int no_abort = 0;
+      for (int gg = (g > S ? g - S : 0); gg < g; ++gg)
+        mbar_wait_warp(&full[gg % S], (gg / S) & 1, &no_abort, a.err, kDevTimeoutDrain);
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
-      // One thread issues every MMA, so the loop body is kept short: descriptors and
-      // TMEM addresses advance by additions, segment boundaries by a countdown.
-      const uint32_t idesc = idesc_e4m3_m128(NT);
-      const int planes = a.planes;
-      // Shared-memory descriptors hold address >> 4 in their low bits, so a byte offset
-      // `o` into a region is `desc + (o >> 4)`.
-      const uint64_t act_desc0 = sdesc_sw128(smem_u32(sm.act(0, 0, 0)));
-      const uint64_t conv_desc0 = kATmem ? 0 : sdesc_sw128(smem_u32(sm.conv(0, 0)));
-      const uint32_t slot_step = (uint32_t)(sm.slot_bytes >> 4);
-      const uint32_t act_step = (uint32_t)(Smem<NT, KPS>::kActBytes >> 4);
-      const uint32_t a_tmem0 = tmem_base + a.a_col0;
-      Ring rg(S), rc(CS);
-      int u = 0, mma_done = 0;
-      while (iter.next(un)) {
-        const int b = a.nbuf == 2 ? (u & 1) : 0;
-        const uint32_t tpar = ((a.nbuf == 2 ? (u >> 1) : u) & 1) ^ 1;
-        if (!mbar_wait(&tempty[b], tpar, abort_flag, a.err, kDevTimeoutTmemEmpty)) break;
+    // The whole warp runs the loop (uniform control flow, warp-wide waits) and one lane,
+    // elected once, issues every MMA and commit: tcgen05 issue from a converged warp's
+    // leader is about twice as fast as from a thread looping alone, and a commit tracks
+    // the MMAs of the thread that issues it.  Descriptors and TMEM addresses advance by
+    // additions, segment boundaries by a countdown.
+    const bool leader = elect_one();
+    const uint32_t idesc = idesc_e4m3_m128(NT);
+    const int planes = a.planes;
+    // Shared-memory descriptors hold address >> 4 in their low bits, so a byte offset
+    // `o` into a region is `desc + (o >> 4)`.
+    const uint64_t act_desc0 = sdesc_sw128(smem_u32(sm.act(0, 0, 0)));
+    const uint64_t conv_desc0 = kATmem ? 0 : sdesc_sw128(smem_u32(sm.conv(0, 0)));
+    const uint32_t slot_step = (uint32_t)(sm.slot_bytes >> 4);
+    const uint32_t act_step = (uint32_t)(Smem<NT, KPS>::kActBytes >> 4);
+    const uint32_t a_tmem0 = tmem_base + a.a_col0;
+    Ring rg(S), rc(CS);
+    int u = 0, mma_done = 0;
+    while (iter.next(un)) {
+      const int b = a.nbuf == 2 ? (u & 1) : 0;
+      const uint32_t tpar = ((a.nbuf == 2 ? (u >> 1) : u) & 1) ^ 1;
+      if (!mbar_wait_warp(&tempty[b], tpar, abort_flag, a.err, kDevTimeoutTmemEmpty)) break;
+      tc_fence_after();
+      uint32_t d = tmem_base + (uint32_t)(b * NT * a.segs);
+      int seg_left = a.seg_iters - un.i0 % a.seg_iters;   // iterations left in this segment
+      uint32_t fresh = 1;
+      bool ok = true;
+      for (int it = un.i0; it < un.i1; ++it, rg.next(), rc.next()) {
+        const int s = rg.s, c = rc.s;
+        if (!mbar_wait_warp(&cfull[c], rc.ph, abort_flag, a.err, kDevTimeoutConv)) {
+          ok = false;
+          break;
+        }
+        const int gm = it - un.i0 + mma_done;
+        if (leader && gm < 16) DPTQ_TRACE_POINT(tr, 72 + gm);
         tc_fence_after();
-        uint32_t d = tmem_base + (uint32_t)(b * NT * a.segs);
-        int seg_left = a.seg_iters - un.i0 % a.seg_iters;   // iterations left in this segment
-        uint32_t fresh = 1;
-        bool ok = true;
-        for (int it = un.i0; it < un.i1; ++it, rg.next(), rc.next()) {
-          const int s = rg.s, c = rc.s;
-          if (!mbar_wait(&cfull[c], rc.ph, abort_flag, a.err, kDevTimeoutConv)) {
-            ok = false;
-            break;
-          }
-          const int gm = it - un.i0 + mma_done;
-          if (gm < 16) DPTQ_TRACE_POINT(tr, 72 + gm);
-          tc_fence_after();
-          if (seg_left == 0) {   // next exact-accumulation segment: next accumulator
-            d += NT;
-            fresh = 1;
-            seg_left = a.seg_iters;
-          }
-          const uint64_t bd_slot = act_desc0 + (uint64_t)(s * slot_step);
+        if (seg_left == 0) {   // next exact-accumulation segment: next accumulator
+          d += NT;
+          fresh = 1;
+          seg_left = a.seg_iters;
+        }
+        const uint64_t bd_slot = act_desc0 + (uint64_t)(s * slot_step);
+        if (leader) {
 #pragma unroll
           for (int h = 0; h < KPS; ++h) {
             const uint64_t ad = conv_desc0 + (uint64_t)((c * KPS + h) * (kConvBytes >> 4));
@@ -340,19 +351,22 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
           mma_commit(&empty[s]);
           mma_commit(&cempty[c]);
           if (gm < 16) DPTQ_TRACE_POINT(tr, 88 + gm);
-          fresh = 0;
-          --seg_left;
         }
-        if (!ok) break;
-        mma_commit(&tfull[b]);
-        mma_done += un.i1 - un.i0;
-        ++u;
+        __syncwarp();
+        fresh = 0;
+        --seg_left;
       }
-      // Every MMA this thread issued must be complete before TMEM is released.
-      mma_commit(drain);
-      volatile int no_abort = 0;
-      mbar_wait(drain, 0, &no_abort, a.err, kDevTimeoutDrain);
+      if (!ok) break;
+      if (leader) mma_commit(&tfull[b]);
+      __syncwarp();
+      mma_done += un.i1 - un.i0;
+      ++u;
     }
+    // Every MMA the leader issued must be complete before TMEM is released.
+    if (leader) mma_commit(drain);
+    __syncwarp();
+    volatile int no_abort = 0;
+    mbar_wait_warp(drain, 0, &no_abort, a.err, kDevTimeoutDrain);
   } else if (warp < kEpiWarp0) {
     // ------------------------------------------------------------ converters
     const int ctid = threadIdx.x - kConvWarp0 * 32;   // 0..255
