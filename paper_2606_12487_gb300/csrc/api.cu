@@ -175,6 +175,7 @@ dptq_status run_gemm(dptq_handle h, const GemmPlan& plan0, const uint8_t* act, c
   g.sa = sa;
   g.sw = h->sw;
   g.out = static_cast<__half*>(out);
+  g.out_vec = (reinterpret_cast<uintptr_t>(out) & 15u) == 0;
   g.acc_out = acc;
   g.ws = sc->ws;
   g.counters = sc->counters;

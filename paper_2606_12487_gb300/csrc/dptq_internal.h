@@ -91,6 +91,7 @@ struct GemmArgs {
   int dp_tiles;        // tiles processed whole, round-robin, before the stream-K part
   long long sk_iters;  // stream-K iterations (tiles after dp_tiles, times KI)
   uint32_t tmem_cols;
+  int out_vec;         // `out` is 16-byte aligned: the epilogue stores 8 channels at a time
 };
 
 struct GemmPlan {

@@ -48,7 +48,7 @@ constexpr int kConvBytes = 128 * 128;   // one weight tile widened to E4M3
 constexpr int kMaxStages = 8;
 constexpr int kMaxConvSlots = 4;
 constexpr int kSmemLimit = 232448;      // 227 KB opt-in dynamic shared memory per CTA
-constexpr int kBarrierBytes = 1024;
+constexpr int kBarrierBytes = 2048;   // barriers and flags, token scales (tiles <= 64), output transpose (1 KB)
 
 struct Unit {
   int tile;
@@ -58,45 +58,46 @@ struct Unit {
 };
 
 // Deterministic enumeration of one CTA's work; every warp role walks the same list.
+// The stream-K part spans fewer than 2 * G * KI iterations (at most 2G tiles are left
+// after the data-parallel rounds), so all products below fit in 32 bits (the planner
+// checks this); 32-bit divisions keep the per-unit cost low.
 struct UnitIter {
-  int cta, G, KI, dp_tiles, dp_next;
-  long long sk_iters, it, it_end;
+  uint32_t cta, G, KI, dp_tiles, dp_next;
+  uint32_t sk_iters, it, it_end;
 
-  __device__ __forceinline__ long long sk_begin(int c) const { return ((long long)c * sk_iters) / G; }
-  __device__ __forceinline__ int cta_of(long long i) const {
-    return (int)(((i + 1) * (long long)G - 1) / sk_iters);
-  }
+  __device__ __forceinline__ uint32_t sk_begin(uint32_t c) const { return (c * sk_iters) / G; }
+  __device__ __forceinline__ uint32_t cta_of(uint32_t i) const { return ((i + 1) * G - 1) / sk_iters; }
   __device__ __forceinline__ void init(const GemmArgs& a) {
     cta = blockIdx.x;
     G = gridDim.x;
-    KI = a.KI;
-    dp_tiles = a.dp_tiles;
+    KI = (uint32_t)a.KI;
+    dp_tiles = (uint32_t)a.dp_tiles;
     dp_next = cta;
-    sk_iters = a.sk_iters;
+    sk_iters = (uint32_t)a.sk_iters;
     it = sk_iters > 0 ? sk_begin(cta) : 0;
     it_end = sk_iters > 0 ? sk_begin(cta + 1) : 0;
   }
   __device__ __forceinline__ bool next(Unit& u) {
     if (dp_next < dp_tiles) {
-      u.tile = dp_next;
+      u.tile = (int)dp_next;
       u.i0 = 0;
-      u.i1 = KI;
+      u.i1 = (int)KI;
       u.slot = -1;
       u.contributors = 1;
       dp_next += G;
       return true;
     }
     if (it >= it_end) return false;
-    const long long t = it / KI;
-    const int i0 = (int)(it - t * KI);
-    const long long left = it_end - it;
-    const int i1 = (int)((long long)(KI - i0) < left ? KI : i0 + left);
-    const int c0 = cta_of(t * KI), c1 = cta_of(t * KI + KI - 1);
-    u.tile = dp_tiles + (int)t;
-    u.i0 = i0;
-    u.i1 = i1;
-    u.slot = (c0 == c1) ? -1 : c0;
-    u.contributors = c1 - c0 + 1;
+    const uint32_t t = it / KI;
+    const uint32_t i0 = it - t * KI;
+    const uint32_t left = it_end - it;
+    const uint32_t i1 = KI - i0 < left ? KI : i0 + left;
+    const uint32_t c0 = cta_of(t * KI), c1 = cta_of(t * KI + KI - 1);
+    u.tile = (int)(dp_tiles + t);
+    u.i0 = (int)i0;
+    u.i1 = (int)i1;
+    u.slot = (c0 == c1) ? -1 : (int)c0;
+    u.contributors = (int)(c1 - c0 + 1);
     it += i1 - i0;
     return true;
   }
@@ -171,12 +172,15 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
   uint64_t* esync = drain + 1;   // epilogue-group barrier (4 warps), bounded waits
   uint32_t* tmem_base_sh = reinterpret_cast<uint32_t*>(esync + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_base_sh + 1);
-  volatile int* last_flag = reinterpret_cast<volatile int*>(tmem_base_sh + 2);
+  volatile int* flags = reinterpret_cast<volatile int*>(tmem_base_sh + 2);   // epilogue: 2 units x 2
+  float* sa_sh = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + 512);   // token scales (NT <= 64)
+  __half* xpose = reinterpret_cast<__half*>(reinterpret_cast<uint8_t*>(bars) + 1024);  // 4 x [4 tokens][32 ch]
   const uint8_t** pend_src = reinterpret_cast<const uint8_t**>(tmem_base_sh + 8);   // producer's pending list
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   unsigned long long* const tr = DPTQ_TRACE_BUF();
+  (void)tr;
   if (threadIdx.x == 0) DPTQ_TRACE_POINT(tr, 0);
 
   if (threadIdx.x == 0) {
@@ -195,7 +199,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
     mbar_init(drain, 1);
     mbar_init(esync, kNumEpiWarps);
     *abort_flag = 0;
-    *last_flag = 0;
+    for (int i = 0; i < 4; ++i) flags[i] = 0;
     fence_mbar_init();
   }
   if (warp == 1) {
@@ -217,6 +221,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
     // ------------------------------------------------------------ producer
     // Whole warp, uniform control flow; the elected leader issues the copies.
     const bool leader = elect_one();
+    if (leader) DPTQ_TRACE_POINT(tr, 117);
     const uint64_t pol_w = l2_policy_evict_first();   // weights are streamed once
     const uint64_t pol_a = l2_policy_evict_last();    // activations are re-read per n-tile
     const uint32_t act_bytes = (uint32_t)NT * 128;
@@ -241,6 +246,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
     while (ok && iter.next(un)) {
       const int nt = un.tile / a.m_tiles;
       const int mt = un.tile - nt * a.m_tiles;
+      if (leader) DPTQ_TRACE_POINT(tr, 118);
       const uint8_t* wsrc = a.wt + ((size_t)nt * a.KB + (size_t)un.i0 * KPS) * kWTileBytes;
       const uint8_t* asrc = a.act + ((size_t)un.i0 * KPS * a.M_pad + (size_t)mt * NT) * 128;
       for (int it = un.i0; it < un.i1; ++it, ++g, rg.next(), wsrc += w_bytes, asrc += KPS * kb_stride) {
@@ -462,96 +468,198 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
       ++esync_phase;
       return ok;
     };
+    int sa_mt = -1;   // token tile whose activation scales sit in sa_sh
     int u = 0;
     while (iter.next(un)) {
       const int b = a.nbuf == 2 ? (u & 1) : 0;
       const uint32_t tpar = (a.nbuf == 2 ? (u >> 1) : u) & 1;
-      if (!mbar_wait(&tfull[b], tpar, abort_flag, a.err, kDevTimeoutTmemFull)) break;
-      if (etid == 0 && u < 4) DPTQ_TRACE_POINT(tr, 104 + u);
-      tc_fence_after();
       const int nt = un.tile / a.m_tiles;
       const int mt = un.tile - nt * a.m_tiles;
       const int n = nt * 128 + q * 32 + lane;
       const int m0 = mt * NT;
+      // Scales are fetched while the MMAs of this unit still run.
+      const float swn = n < a.N ? sw_g[n] : 0.f;
+      if (NT <= 64 && mt != sa_mt) {
+        if (!epi_sync()) break;   // every warp is done with the previous token tile's scales
+        for (int i = etid; i < NT; i += kNumEpiWarps * 32) sa_sh[i] = m0 + i < a.M ? sa_g[m0 + i] : 0.f;
+        if (!epi_sync()) break;
+        sa_mt = mt;
+      }
+      if (!mbar_wait(&tfull[b], tpar, abort_flag, a.err, kDevTimeoutTmemFull)) break;
+      if (etid == 0 && u < 4) DPTQ_TRACE_POINT(tr, 104 + u);
+      tc_fence_after();
       const int nseg = (un.i1 - 1) / a.seg_iters - un.i0 / a.seg_iters + 1;
       const uint32_t tb = tmem_base + lane_base + (uint32_t)(b * NT * a.segs);
-      const float swn = n < a.N ? sw_g[n] : 0.f;
       int32_t* __restrict__ wsl = un.slot >= 0 ? ws_g + (size_t)un.slot * (NT * 128) : nullptr;
+      // Split tile.  If every other contributor has already added its part to the slot,
+      // this CTA finishes the tile straight from its accumulators (slot + own part);
+      // otherwise it adds its part and the last contributor to arrive finishes.
+      volatile int* const flag = flags + 2 * (u & 1);   // [0]: all others in, [1]: last
+      bool finish = wsl == nullptr;
+      if (wsl != nullptr) {
+        if (etid == 0) *flag = ld_acquire_gpu(a.counters + un.slot) == (uint32_t)(un.contributors - 1);
+        if (!epi_sync()) break;
+        finish = *flag != 0;
+        if (etid == 0) DPTQ_TRACE_POINT(tr, 3);
+      }
+      // Output of 16 tokens of this thread's channel.  With a 16-byte aligned `out`, each
+      // warp transposes 4 tokens x 32 channels at a time through shared memory and every
+      // lane stores 4 consecutive channels of one token (8 bytes instead of four 2-byte
+      // stores).  Token scales come from shared memory for tiles of up to 64 tokens, else
+      // from the (cached) global array.
+      auto write_out = [&](int c0, const int (&v)[16]) {
+        __half hv[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int m = m0 + c0 + i;
+          const float sav = NT <= 64 ? sa_sh[c0 + i] : (m < a.M ? __ldg(sa_g + m) : 0.f);
+          hv[i] = __float2half_rn(__fmul_rn(__fmul_rn(__int2float_rn(v[i]), sav), swn));
+        }
+        if (acc_g != nullptr && n < a.N) {
+#pragma unroll
+          for (int i = 0; i < 16; ++i)
+            if (m0 + c0 + i < a.M) acc_g[(size_t)(m0 + c0 + i) * a.N + n] = v[i];
+        }
+        if (a.out_vec) {
+          __half* xw = xpose + q * 128;
+          const int c = lane >> 3;                 // token of this lane's 8-byte store
+          const int nn = nt * 128 + q * 32 + (lane & 7) * 4;
+#pragma unroll
+          for (int g4 = 0; g4 < 4; ++g4) {
+#pragma unroll
+            for (int i = 0; i < 4; ++i) xw[i * 32 + lane] = hv[4 * g4 + i];
+            __syncwarp();
+            const uint2 val = *reinterpret_cast<const uint2*>(xw + c * 32 + (lane & 7) * 4);
+            __syncwarp();
+            const int m = m0 + c0 + 4 * g4 + c;
+            if (m < a.M && nn < a.N) *reinterpret_cast<uint2*>(out_g + (size_t)m * a.N + nn) = val;
+          }
+        } else if (n < a.N) {
+#pragma unroll
+          for (int i = 0; i < 16; ++i)
+            if (m0 + c0 + i < a.M) out_g[(size_t)(m0 + c0 + i) * a.N + n] = hv[i];
+        }
+      };
+      // Split-tile partial sums.  With one exact-accumulation segment (every partial
+      // sum and every sum of partial sums is an integer multiple of 2^-9 below 2^24
+      // units, so exact in fp32) the raw fp32 accumulators are added with vector
+      // reductions into a slot laid out [token / 4][channel][token % 4] (a warp's vector
+      // access covers 512 contiguous bytes); otherwise int32 atomics, token-major.
+      const bool f32 = a.segs == 1;
+      float* const wslf = wsl != nullptr ? reinterpret_cast<float*>(wsl) + (size_t)(q * 32 + lane) * 4 : nullptr;
 #pragma unroll 1
       for (int c0 = 0; c0 < NT; c0 += 16) {
         int acc[16];
+        if (f32) {
+          float f[16];
+          if (finish && wsl != nullptr) {
 #pragma unroll
-        for (int i = 0; i < 16; ++i) acc[i] = 0;
-        for (int sg = 0; sg < nseg; ++sg) {
-          uint32_t r[16];
-          tmem_ld16(tb + (uint32_t)(sg * NT + c0), r);
-          tmem_ld_wait();
-#pragma unroll
-          for (int i = 0; i < 16; ++i) acc[i] += __float2int_rn(__uint_as_float(r[i]) * 512.f);
-        }
-        if (wsl == nullptr) {
-          float sav[16];
-#pragma unroll
-          for (int i = 0; i < 16; ++i) sav[i] = (m0 + c0 + i < a.M) ? sa_g[m0 + c0 + i] : 0.f;
-          if (n < a.N) {
-#pragma unroll
-            for (int i = 0; i < 16; ++i) {
-              const int m = m0 + c0 + i;
-              if (m < a.M) {
-                const float t = __fmul_rn(__int2float_rn(acc[i]), sav[i]);
-                out_g[(size_t)m * a.N + n] = __float2half_rn(__fmul_rn(t, swn));
-                if (acc_g) acc_g[(size_t)m * a.N + n] = acc[i];
-              }
+            for (int j = 0; j < 4; ++j) {
+              const float4 t = __ldcg(reinterpret_cast<const float4*>(wslf + (c0 / 4 + j) * 512));
+              f[4 * j] = t.x;
+              f[4 * j + 1] = t.y;
+              f[4 * j + 2] = t.z;
+              f[4 * j + 3] = t.w;
             }
+#pragma unroll
+            for (int j = 0; j < 4; ++j)   // zero for the next launch
+              __stcg(reinterpret_cast<float4*>(wslf + (c0 / 4 + j) * 512), make_float4(0.f, 0.f, 0.f, 0.f));
+          } else {
+#pragma unroll
+            for (int i = 0; i < 16; ++i) f[i] = 0.f;
+          }
+          uint32_t r[16];
+          tmem_ld16(tb + (uint32_t)c0, r);
+          tmem_ld_wait();
+          if (etid == 0 && c0 == 0) DPTQ_TRACE_POINT(tr, 2);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) f[i] = __fadd_rn(f[i], __uint_as_float(r[i]));
+          if (etid == 0) DPTQ_TRACE_POINT(tr, c0 == 0 ? 4 : 119);
+          if (finish) {
+#pragma unroll
+            for (int i = 0; i < 16; ++i) acc[i] = __float2int_rn(f[i] * 512.f);
+            write_out(c0, acc);
+          } else {
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+              red_add_v4_f32(wslf + (c0 / 4 + j) * 512, f[4 * j], f[4 * j + 1], f[4 * j + 2], f[4 * j + 3]);
           }
         } else {
+          if (finish && wsl != nullptr) {
 #pragma unroll
-          for (int i = 0; i < 16; ++i) atomicAdd(wsl + (c0 + i) * 128 + q * 32 + lane, acc[i]);
+            for (int i = 0; i < 16; ++i) acc[i] = __ldcg(wsl + (c0 + i) * 128 + q * 32 + lane);
+#pragma unroll
+            for (int i = 0; i < 16; ++i) __stcg(wsl + (c0 + i) * 128 + q * 32 + lane, 0);   // zero for the next launch
+          } else {
+#pragma unroll
+            for (int i = 0; i < 16; ++i) acc[i] = 0;
+          }
+          for (int sg = 0; sg < nseg; ++sg) {
+            uint32_t r[16];
+            tmem_ld16(tb + (uint32_t)(sg * NT + c0), r);
+            tmem_ld_wait();
+#pragma unroll
+            for (int i = 0; i < 16; ++i) acc[i] += __float2int_rn(__uint_as_float(r[i]) * 512.f);
+          }
+          if (finish) {
+            write_out(c0, acc);
+          } else {
+#pragma unroll
+            for (int i = 0; i < 16; ++i) atomicAdd(wsl + (c0 + i) * 128 + q * 32 + lane, acc[i]);
+          }
         }
+        if (etid == 0) DPTQ_TRACE_POINT(tr, c0 == 0 ? 6 : 123);
       }
       if (etid == 0 && u < 4) DPTQ_TRACE_POINT(tr, 112 + u);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&tempty[b]);
       ++u;
-      if (wsl != nullptr) {
-        // Split tile: publish this CTA's part, and let the last contributor finish.
+      if (wsl != nullptr && finish) {
+        if (etid == 0) a.counters[un.slot] = 0u;   // every other contributor has arrived
+      } else if (wsl != nullptr) {
+        // Publish this CTA's part; the contributor that arrives last finishes the tile.
         __threadfence();
         if (!epi_sync()) break;
         if (etid == 0) {
-          const unsigned prev = atomicAdd(a.counters + un.slot, 1u);
-          const int last = prev == (unsigned)(un.contributors - 1);
-          if (last) a.counters[un.slot] = 0u;   // every contributor has arrived
-          *last_flag = last;
+          const uint32_t prev = atom_add_acq_rel_gpu(a.counters + un.slot, 1u);
+          const int last = prev == (uint32_t)(un.contributors - 1);
+          if (last) a.counters[un.slot] = 0u;
+          flag[1] = last;
+          DPTQ_TRACE_POINT(tr, 5);
         }
         if (!epi_sync()) break;
-        if (*last_flag) {
-          __threadfence();
+        if (flag[1]) {
 #pragma unroll 1
           for (int c0 = 0; c0 < NT; c0 += 16) {
             int v[16];
-            float sav[16];
+            if (f32) {
 #pragma unroll
-            for (int i = 0; i < 16; ++i) v[i] = __ldcg(wsl + (c0 + i) * 128 + q * 32 + lane);
-#pragma unroll
-            for (int i = 0; i < 16; ++i) sav[i] = (m0 + c0 + i < a.M) ? sa_g[m0 + c0 + i] : 0.f;
-#pragma unroll
-            for (int i = 0; i < 16; ++i) __stcg(wsl + (c0 + i) * 128 + q * 32 + lane, 0);   // zeroed for the next launch
-            if (n < a.N) {
-#pragma unroll
-              for (int i = 0; i < 16; ++i) {
-                const int m = m0 + c0 + i;
-                if (m < a.M) {
-                  const float t = __fmul_rn(__int2float_rn(v[i]), sav[i]);
-                  out_g[(size_t)m * a.N + n] = __float2half_rn(__fmul_rn(t, swn));
-                  if (acc_g) acc_g[(size_t)m * a.N + n] = v[i];
-                }
+              for (int j = 0; j < 4; ++j) {
+                const float4 t = __ldcg(reinterpret_cast<const float4*>(wslf + (c0 / 4 + j) * 512));
+                v[4 * j] = __float2int_rn(t.x * 512.f);
+                v[4 * j + 1] = __float2int_rn(t.y * 512.f);
+                v[4 * j + 2] = __float2int_rn(t.z * 512.f);
+                v[4 * j + 3] = __float2int_rn(t.w * 512.f);
               }
+#pragma unroll
+              for (int j = 0; j < 4; ++j)
+                __stcg(reinterpret_cast<float4*>(wslf + (c0 / 4 + j) * 512), make_float4(0.f, 0.f, 0.f, 0.f));
+            } else {
+#pragma unroll
+              for (int i = 0; i < 16; ++i) v[i] = __ldcg(wsl + (c0 + i) * 128 + q * 32 + lane);
+#pragma unroll
+              for (int i = 0; i < 16; ++i) __stcg(wsl + (c0 + i) * 128 + q * 32 + lane, 0);
             }
+            write_out(c0, v);
           }
         }
-        if (!epi_sync()) break;
+        if (etid == 0) {
+          DPTQ_TRACE_POINT(tr, 7);
+          DPTQ_TRACE_VALUE(tr, 121, flag[1] + 2);
+        }
       }
+      if (wsl != nullptr && finish && etid == 0) DPTQ_TRACE_VALUE(tr, 121, 1);
       if (etid == 0 && u <= 4) DPTQ_TRACE_POINT(tr, 108 + u - 1);
     }
     if (etid == 0) DPTQ_TRACE_VALUE(tr, 122, u);
@@ -662,7 +770,10 @@ bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan) {
   a.conv_slots = conv_slots;
   a.dp_tiles = (int)dp;
   a.sk_iters = (tiles - dp) * KI;
+  // 32-bit work enumeration on the device (UnitIter).
+  if ((long long)a.sk_iters * G + G >= (1LL << 32) || tiles >= (1LL << 31)) return false;
   a.tmem_cols = cols;
+  a.out_vec = 0;
   return true;
 }
 

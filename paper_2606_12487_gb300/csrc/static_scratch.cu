@@ -155,6 +155,7 @@ extern "C" dptq_status dptq_qlinear_static(dptq_handle h, const void* x_fp16, in
   g.sa = sa;
   g.sw = h->sw;
   g.out = static_cast<__half*>(out_fp16);
+  g.out_vec = (reinterpret_cast<uintptr_t>(out_fp16) & 15u) == 0;
   g.acc_out = nullptr;
   g.ws = reinterpret_cast<int32_t*>(st->base + kWsOff);
   g.counters = reinterpret_cast<uint32_t*>(st->base + kCntOff);

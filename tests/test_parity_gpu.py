@@ -227,6 +227,27 @@ def test_qlinear_edge_inputs(dp, orc):
         assert np.all(got[0] == 0) and np.all(got[:, 3] == 0)
 
 
+@pytest.mark.parametrize("M,N,K,B", [(17, 272, 1024, 1024), (32, 4096, 4096, 4096)])
+def test_qlinear_unaligned_output(dp, M, N, K, B):
+    """An output pointer that is not 16-byte aligned takes the scalar-store epilogue;
+    it must give the same bits as an aligned one (split tiles included)."""
+    wl = inputs.llama2_7b_decode()
+    x = torch.from_numpy(inputs.activations(wl, M, K)).to(DEV)
+    W = inputs.weights(N, K, layer=2, proj=3)
+    layer = dp.dptq_pack_weights(torch.from_numpy(W).to(DEV), B)
+    for bits in (4, 8):
+        ref = torch.empty((M, N), dtype=torch.float16, device=DEV)
+        dp.dptq_qlinear(layer, x, bits, ref)
+        flat = torch.zeros(M * N + 8, dtype=torch.float16, device=DEV)
+        out = flat[1:1 + M * N].view(M, N)
+        assert out.data_ptr() % 16 != 0
+        dp.dptq_qlinear(layer, x, bits, out)
+        torch.cuda.synchronize()
+        assert torch.equal(out.view(torch.int16), ref.view(torch.int16))
+        assert flat[0].item() == 0 and torch.all(flat[1 + M * N:] == 0)
+    layer.close()
+
+
 def test_qlinear_m_zero_is_noop(dp):
     W = inputs.weights(128, 256)
     layer = dp.dptq_pack_weights(torch.from_numpy(W).to(DEV), 256)
