@@ -157,9 +157,10 @@ def _inputs():
 
 
 class Stack:
-    def __init__(self, dp, wl, layers, M, device):
+    def __init__(self, dp, wl, layers, M, device, path="fused"):
         import torch
         self.dp, self.wl, self.layers, self.M = dp, wl, layers, M
+        self.path = path   # "fused": one dptq_qlinear launch per projection; "split": quantize + GEMM
         groups = stack_groups(wl)
         self.x = [torch.from_numpy(_inputs().activations(wl, M, K, seed=gi)).to(device)
                   for gi, (_, K, _, _, _) in enumerate(groups)]
@@ -173,6 +174,15 @@ class Stack:
         for li, hs in enumerate(self.layers):
             bits = self.wl.bits(li)
             for gi, h in enumerate(hs):
+                if self.path == "fused":
+                    if gemm_events is not None:
+                        e0, e1 = gemm_events.pop()
+                        e0.record(stream)
+                    dp.dptq_qlinear(h, self.x[gi], bits, self.out[gi], stream=stream)
+                    if gemm_events is not None:
+                        e1.record(stream)
+                        gemm_events_done.append((e0, e1, self.gemm_bytes(gi, bits), self.gemm_ops(gi)))
+                    continue
                 dp.dptq_qlinear_quantize(h, self.x[gi], bits, stream=stream)
                 if gemm_events is not None:
                     e0, e1 = gemm_events.pop()
@@ -184,18 +194,20 @@ class Stack:
                     dp.dptq_qlinear_gemm(h, self.M, bits, self.out[gi], stream=stream)
 
     def gemm_bytes(self, gi, bits):
-        """Algorithmic HBM bytes of one GEMM launch: packed int4 weights, weight scales,
-        activation codes at b bits, token scales, fp16 output."""
+        """Algorithmic HBM bytes of one timed launch: packed int4 weights, weight scales and
+        the fp16 output, plus the fp16 activations (fused launch) or the activation codes
+        at b bits and token scales (GEMM launch of the split path)."""
         _, K, N, _, _ = self.groups[gi]
         M = self.M
-        return N * K // 2 + 4 * N + M * K * bits // 8 + 4 * M + 2 * M * N
+        act = 2 * M * K if self.path == "fused" else M * K * bits // 8 + 4 * M
+        return N * K // 2 + 4 * N + act + 2 * M * N
 
     def gemm_ops(self, gi):
         _, K, N, _, _ = self.groups[gi]
         return 2 * self.M * N * K
 
     def step_launches(self):
-        return 2 * len(self.groups) * len(self.layers)
+        return (1 if self.path == "fused" else 2) * len(self.groups) * len(self.layers)
 
     def h2d_bytes(self):
         return sum(x.numel() * 2 for x in self.x)
@@ -207,19 +219,28 @@ class Stack:
 gemm_events_done = []
 
 
-def traffic_record():
-    """DRAM bytes / algorithmic bytes of the GEMM from the committed ncu summary, if the
-    summary was taken on the current kernel source (else None)."""
-    import glob
+def kernel_source_sha():
+    """sha256/16 of the sources the timed kernel is compiled from."""
     import hashlib
-    src = os.path.join(ROOT, "paper_2606_12487_gb300", "csrc", "qgemm.cu")
-    try:
-        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
-    except OSError:
+    h = hashlib.sha256()
+    for f in ("qgemm.cu", "rotate_row.cuh", "dptq_device.cuh"):
+        try:
+            h.update(open(os.path.join(ROOT, "paper_2606_12487_gb300", "csrc", f), "rb").read())
+        except OSError:
+            return None
+    return h.hexdigest()[:16]
+
+
+def traffic_record(path_name):
+    """DRAM bytes / algorithmic bytes of the timed kernel from the committed ncu summary,
+    if the summary was taken on the current kernel sources and launch path (else None)."""
+    import glob
+    sha = kernel_source_sha()
+    if sha is None:
         return None
     for path in sorted(glob.glob(os.path.join(ROOT, "profiles", "*.md"))):
         for ln in open(path):
-            if ln.startswith("traffic_record:") and f"sha256/16={sha}" in ln:
+            if ln.startswith("traffic_record:") and f"sha256/16={sha}" in ln and f"path={path_name}" in ln:
                 kv = dict(p.split("=", 1) for p in ln.split() if "=" in p)
                 return int(kv["dram_bytes"]) / int(kv["algorithmic_bytes"]), os.path.basename(path)
     return None
@@ -440,6 +461,9 @@ def main(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--eager", action="store_true",
                     help="launch the step's kernels directly instead of replaying a CUDA graph")
+    ap.add_argument("--path", default="fused", choices=["fused", "split"],
+                    help="fused: one launch per projection (rotation + quantization + GEMM); "
+                         "split: rotate-quantize launch, then GEMM launch")
     ap.add_argument("--layers", type=int, default=0,
                     help="run only the first L layers (small cases for profiler captures; 0 = all)")
     args = ap.parse_args(argv)
@@ -465,7 +489,7 @@ def main(argv=None):
     dptq.dptq_reserve(max_m, max_k, 0)
     stream = torch.cuda.Stream(device=device)
 
-    stack = Stack(dptq, wl, layers, args.m, device)
+    stack = Stack(dptq, wl, layers, args.m, device, args.path)
     g = capture(stack, stream, args.eager)
     ms, clocks = time_graph(g, stream, args.steps, args.warmup, world, local)
     ms_max = max_over_ranks(ms, world, device)
@@ -480,14 +504,14 @@ def main(argv=None):
         pass
     hbm_peak = float(peaks.get("hbm_gbs", 6800.0))
     achieved = tb / tt / 1e9
-    rec = traffic_record()
+    rec = traffic_record(args.path)
     traffic = rec[0] * tb / n_gemm if rec else None
     e2e_dev_s, e2e_wall_s = e2e_measure(stack, g, stream, max(10, args.steps // 4), world)
     e2e_s = max_over_ranks(e2e_dev_s, world, device)
 
     sweep = {}
     for m in [int(v) for v in args.sweep.split(",") if v]:
-        st = Stack(dptq, wl, layers, m, device)
+        st = Stack(dptq, wl, layers, m, device, args.path)
         gm = capture(st, stream, args.eager)
         ms_m, _ = time_graph(gm, stream, max(20, args.steps // 2), args.warmup, world, local, sample_clocks=False)
         ms_m = max_over_ranks(ms_m, world, device)
@@ -509,9 +533,12 @@ def main(argv=None):
         "config": {"workload": f"llama2-7b decode projection stack, {wl.layers} layers, M={args.m} tokens, "
                                "A8 on layers {0,1,30,31}", "global_batch": args.m * world, "seq_len": 1,
                    "parallelism": f"replicas x{world}", "l2": "weights 3.24 GB > L2 (streamed every step)",
+                   "path": args.path,
                    "weight_bytes_per_step": weight_bytes},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
-                     "frac": achieved / hbm_peak, "traffic": traffic, "kernel": "qgemm_kernel",
+                     "frac": achieved / hbm_peak, "traffic": traffic,
+                     "kernel": "qgemm_kernel (fused rotation + quantization + GEMM)" if args.path == "fused"
+                               else "qgemm_kernel",
                      "traffic_note": (f"bytes per average launch: ncu DRAM/algorithmic ratio {rec[0]:.3f} "
                                       f"({rec[1]}) x {tb / n_gemm:.0f} algorithmic bytes") if rec else
                                      "no capture of the current kernel source",

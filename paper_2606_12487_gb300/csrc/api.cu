@@ -98,7 +98,8 @@ struct Scratch {
   float* sa = nullptr;
   size_t sa_count = 0;
   int32_t* ws = nullptr;
-  uint32_t* counters = nullptr;
+  uint32_t* counters = nullptr;   // [num_sms] split-tile arrivals, then [2] fused-launch grid counters
+  uint32_t* gsync = nullptr;
   int* err = nullptr;
   int num_sms = 0;
 };
@@ -127,10 +128,11 @@ dptq_status ensure_scratch(int dev, size_t act_bytes, size_t sa_count, cudaStrea
     DPTQ_CUDA(cudaDeviceGetAttribute(&sc.num_sms, cudaDevAttrMultiProcessorCount, dev), "cudaDeviceGetAttribute");
     const size_t ws_bytes = (size_t)sc.num_sms * kMaxNT * 128 * sizeof(int32_t);
     DPTQ_CUDA(cudaMalloc(&sc.ws, ws_bytes), "cudaMalloc(ws)");
-    DPTQ_CUDA(cudaMalloc(&sc.counters, sizeof(uint32_t) * sc.num_sms), "cudaMalloc(counters)");
+    DPTQ_CUDA(cudaMalloc(&sc.counters, sizeof(uint32_t) * (sc.num_sms + 2)), "cudaMalloc(counters)");
+    sc.gsync = sc.counters + sc.num_sms;
     DPTQ_CUDA(cudaMalloc(&sc.err, sizeof(int)), "cudaMalloc(err)");
     DPTQ_CUDA(cudaMemset(sc.ws, 0, ws_bytes), "cudaMemset(ws)");
-    DPTQ_CUDA(cudaMemset(sc.counters, 0, sizeof(uint32_t) * sc.num_sms), "cudaMemset(counters)");
+    DPTQ_CUDA(cudaMemset(sc.counters, 0, sizeof(uint32_t) * (sc.num_sms + 2)), "cudaMemset(counters)");
     DPTQ_CUDA(cudaMemset(sc.err, 0, sizeof(int)), "cudaMemset(err)");
   }
   if (grow_act || grow_sa) DPTQ_CUDA(cudaDeviceSynchronize(), "cudaDeviceSynchronize");
@@ -179,6 +181,7 @@ dptq_status run_gemm(dptq_handle h, const GemmPlan& plan0, const uint8_t* act, c
   g.acc_out = acc;
   g.ws = sc->ws;
   g.counters = sc->counters;
+  g.gsync = sc->gsync;
   g.err = sc->err;
   DPTQ_CUDA(launch_gemm(plan, s, true), "qgemm launch");
   return DPTQ_OK;
@@ -190,6 +193,14 @@ namespace dptq {
 bool pdl_allowed() {
   static const bool on = [] {
     const char* v = std::getenv("DPTQ_PDL");
+    return !(v && v[0] == '0');
+  }();
+  return on;
+}
+
+bool fused_allowed() {
+  static const bool on = [] {
+    const char* v = std::getenv("DPTQ_FUSED");
     return !(v && v[0] == '0');
   }();
   return on;
@@ -326,6 +337,16 @@ dptq_status dptq_qlinear(dptq_handle h, const void* x_fp16, int M, int bits, voi
   dptq_status st = prepare_qlinear(h, M, bits, s, &dev, &plan, &sc);
   if (st != DPTQ_OK || M == 0) return st;
   if (!x_fp16 || !out_fp16) return fail(DPTQ_ERR_INVALID_ARG, "null pointer");
+  // Small M: one launch that rotates and quantizes the rows and runs the GEMM.
+  GemmPlan fp;
+  if (fused_allowed() &&
+      plan_gemm(M, h->N, h->K_pad, bits, sc->num_sms, fp, (int)rotate_quant_smem(h->K, 0)) &&
+      fp.M_pad == plan.M_pad) {
+    int nfull, tail, log2B;
+    if ((st = check_shape(h->K, h->had_block, nfull, tail, log2B)) != DPTQ_OK) return st;
+    fp.args.rq = make_rq(x_fp16, M, fp.M_pad, h->K, h->KB, h->had_block, nfull, tail, log2B, bits, sc->sa, sc->act);
+    return run_gemm(h, fp, sc->act, sc->sa, out_fp16, nullptr, sc, s);
+  }
   if ((st = quantize_into_scratch(h, x_fp16, M, bits, plan, sc, s)) != DPTQ_OK) return st;
   return run_gemm(h, plan, sc->act, sc->sa, out_fp16, nullptr, sc, s);
 }

@@ -10,7 +10,7 @@ namespace dptq {
 
 // ------------------------------------------------------------------ tracing
 // Built with -DDPTQ_TRACE (a separate library, see build.py), kernels record
-// %globaltimer stamps per CTA at fixed slots of a 128-entry row of the buffer set by
+// %globaltimer stamps per CTA at fixed slots of a 256-entry row of the buffer set by
 // dptq_trace_set(); otherwise the trace points compile to nothing.
 #ifdef DPTQ_TRACE
 // One copy per translation unit; dptq_trace_set() sets the GEMM's.
@@ -22,11 +22,11 @@ __device__ __forceinline__ unsigned long long trace_now() {
 }
 #define DPTQ_TRACE_POINT(buf, slot) \
   do {                              \
-    if (buf) (buf)[blockIdx.x * 128 + (slot)] = ::dptq::trace_now(); \
+    if (buf) (buf)[blockIdx.x * 256 + (slot)] = ::dptq::trace_now(); \
   } while (0)
 #define DPTQ_TRACE_VALUE(buf, slot, v) \
   do {                                 \
-    if (buf) (buf)[blockIdx.x * 128 + (slot)] = (unsigned long long)(v); \
+    if (buf) (buf)[blockIdx.x * 256 + (slot)] = (unsigned long long)(v); \
   } while (0)
 #define DPTQ_TRACE_BUF() ::dptq::g_dptq_trace
 #else
@@ -178,6 +178,11 @@ __device__ __forceinline__ void tc_fence_before() {
 __device__ __forceinline__ void tc_fence_after() {
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 }
+// Orders this thread's generic-proxy view of global memory (e.g. data another CTA
+// published, acquired here) before its later async-proxy (bulk copy) accesses.
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
 __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
@@ -274,6 +279,12 @@ __device__ __forceinline__ uint32_t atom_add_acq_rel_gpu(uint32_t* p, uint32_t v
 __device__ __forceinline__ void red_add_v4_f32(float* p, float a, float b, float c, float d) {
   asm volatile("red.relaxed.gpu.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(p), "f"(a), "f"(b), "f"(c), "f"(d)
                : "memory");
+}
+
+// Release-add: this thread's earlier writes, and those it has synchronized with (a CTA
+// barrier), are visible at GPU scope before the addition; no return value.
+__device__ __forceinline__ void release_add_gpu(uint32_t* p, uint32_t v) {
+  asm volatile("fence.acq_rel.gpu;\n\tred.relaxed.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
 
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }

@@ -92,9 +92,15 @@ struct GemmArgs {
   long long sk_iters;  // stream-K iterations (tiles after dp_tiles, times KI)
   uint32_t tmem_cols;
   int out_vec;         // `out` is 16-byte aligned: the epilogue stores 8 channels at a time
+  // Fused decode launches only: the rotation + quantization of the M_pad token rows
+  // (written to `act` / `sa` by the converter warps of CTAs 0, 1, ...) and the two grid
+  // counters [rows ready, CTAs done] that order it before the GEMM (zero between launches).
+  RQArgs rq;
+  uint32_t* gsync;
 };
 
 struct GemmPlan {
+  bool fused;     // rotation + quantization inside the GEMM launch
   int nt;          // token tile (MMA N): 16, 32, 64, 128 or 256
   int kps;         // k-blocks of 128 per pipeline stage (1 or 2)
   int M_pad;
@@ -105,12 +111,16 @@ struct GemmPlan {
 
 // Fills everything in `plan.args` that depends only on shapes; the caller sets the
 // pointers.  Returns false if the shape cannot be run.
-bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan);
+// `rot_smem` > 0 plans the fused decode kernel: that many extra bytes of shared memory
+// for the rotation of one row, two k-blocks per stage; false if it does not fit.
+bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan, int rot_smem = 0);
 cudaError_t launch_gemm(const GemmPlan& plan, cudaStream_t s, bool pdl);
 
 // Programmatic dependent launch is on unless the environment sets DPTQ_PDL=0 (kernels
 // then start only after their predecessor has finished, e.g. for profilers).
 bool pdl_allowed();
+// The fused decode kernel is used unless the environment sets DPTQ_FUSED=0.
+bool fused_allowed();
 
 // Message returned by dptq_last_error_message() on the calling thread.
 void set_error_message(const std::string& m);

@@ -37,6 +37,7 @@
 
 #include "dptq_device.cuh"
 #include "dptq_internal.h"
+#include "rotate_row.cuh"
 
 namespace dptq {
 
@@ -150,7 +151,12 @@ struct Smem {
   __device__ __forceinline__ uint8_t* end(int S) const { return slot(S); }
 };
 
-template <int NT, int KPS>
+// FUSED (decode, two-block stages): the launch first rotates and quantizes the token
+// rows itself.  The converter warps of CTA c handle rows c, c + G, ... and publish them
+// on a grid counter; every producer streams its first weight stages meanwhile and
+// requests activation tiles once all M_pad rows are in; the epilogue reads the token
+// scales after the same point.  The last CTA to finish resets the counters.
+template <int NT, int KPS, bool FUSED>
 __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a) {
   // Two-block stages (token tiles of up to 64, weight streaming) widen the weights
   // straight into tensor memory and feed the MMA's A operand from there; one-block
@@ -162,19 +168,23 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
   const int CS = a.conv_slots;
   const Smem<NT, KPS> sm(smem, a.planes, kATmem ? 0 : CS);
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm.end(S));
-  uint64_t* full = bars;                     // slot s: copies landed
+  uint64_t* full = bars;                     // slot s: weight copies landed
   uint64_t* empty = bars + kMaxStages;       // slot s: MMA done with it
-  uint64_t* cfull = bars + 2 * kMaxStages;   // widened slot c: written
+  uint64_t* afull = bars + 2 * kMaxStages;   // slot s: activation copies landed
+  uint64_t* cfull = bars + 3 * kMaxStages;   // widened slot c: written
   uint64_t* cempty = cfull + kMaxConvSlots;  // widened slot c: MMA done with it
   uint64_t* tfull = cempty + kMaxConvSlots;
   uint64_t* tempty = tfull + 2;
   uint64_t* drain = tempty + 2;
   uint64_t* esync = drain + 1;   // epilogue-group barrier (4 warps), bounded waits
-  uint32_t* tmem_base_sh = reinterpret_cast<uint32_t*>(esync + 1);
+  uint64_t* aready = esync + 1;  // fused: all token rows are quantized (producer -> epilogue)
+  uint32_t* tmem_base_sh = reinterpret_cast<uint32_t*>(aready + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_base_sh + 1);
   volatile int* flags = reinterpret_cast<volatile int*>(tmem_base_sh + 2);   // epilogue: 2 units x 2
   float* sa_sh = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + 512);   // token scales (NT <= 64)
   __half* xpose = reinterpret_cast<__half*>(reinterpret_cast<uint8_t*>(bars) + 1024);  // 4 x [4 tokens][32 ch]
+  float* rot_red = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + 768);   // fused: 8 warp maxima
+  unsigned char* rot_smem = reinterpret_cast<unsigned char*>(bars) + kBarrierBytes;    // fused: one row's scratch
   const uint8_t** pend_src = reinterpret_cast<const uint8_t**>(tmem_base_sh + 8);   // producer's pending list
 
   const int warp = threadIdx.x >> 5;
@@ -187,6 +197,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
     for (int s = 0; s < S; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
+      mbar_init(&afull[s], 1);
     }
     for (int c = 0; c < CS; ++c) {
       mbar_init(&cfull[c], kNumConvWarps);
@@ -198,6 +209,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
     }
     mbar_init(drain, 1);
     mbar_init(esync, kNumEpiWarps);
+    mbar_init(aready, 1);
     *abort_flag = 0;
     for (int i = 0; i < 4; ++i) flags[i] = 0;
     fence_mbar_init();
@@ -226,18 +238,52 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
     const uint64_t pol_a = l2_policy_evict_last();    // activations are re-read per n-tile
     const uint32_t act_bytes = (uint32_t)NT * 128;
     const uint32_t w_bytes = (uint32_t)KPS * kWTileBytes;
-    const uint32_t tx = w_bytes + (uint32_t)(KPS * a.planes) * act_bytes;
+    const uint32_t a_tx = (uint32_t)(KPS * a.planes) * act_bytes;
     const size_t plane_stride = (size_t)a.KB * a.M_pad * 128;
     const size_t kb_stride = (size_t)a.M_pad * 128;
     auto issue_act = [&](int slot, const uint8_t* src) {
+      mbar_arrive_expect_tx(&afull[slot], a_tx);
 #pragma unroll
       for (int h = 0; h < KPS; ++h)
         for (int pl = 0; pl < a.planes; ++pl)
-          bulk_g2s(sm.act(slot, h, pl), src + h * kb_stride + pl * plane_stride, act_bytes, &full[slot], pol_a);
+          bulk_g2s(sm.act(slot, h, pl), src + h * kb_stride + pl * plane_stride, act_bytes, &afull[slot], pol_a);
+    };
+    // Activation tiles may be requested once the previous kernel has finished
+    // (programmatic dependent launch) and, in a fused launch, every token row has been
+    // quantized.  False only when the CTA aborts.
+    auto act_ready = [&]() -> bool {
+      pdl_wait();
+      if constexpr (FUSED) {
+        const long long t0 = clock64();
+        while (true) {
+          int st = 0;
+          if (lane == 0) {
+            if (ld_acquire_gpu(a.gsync) >= (uint32_t)a.M_pad)
+              st = 1;
+            else if (*abort_flag)
+              st = 2;
+            else if (clock64() - t0 > kWaitTimeoutCycles) {
+              *abort_flag = 1;
+              atomicCAS(a.err, 0, (int)kDevTimeoutGrid);
+              st = 2;
+            }
+          }
+          st = __shfl_sync(0xffffffffu, st, 0);
+          if (st == 1) break;
+          if (st == 2) return false;
+          __nanosleep(32);
+        }
+        fence_proxy_async_global();   // the bulk copies read what other CTAs stored
+        if (leader) {
+          DPTQ_TRACE_POINT(tr, 116);
+          mbar_arrive(aready);
+        }
+      }
+      return true;
     };
     // Weight tiles do not depend on the previous kernel; the first `S` stages are
-    // requested before waiting for it (programmatic dependent launch) and their
-    // activation halves are issued once the previous kernel has finished.
+    // requested before waiting for it and their activation halves are issued once
+    // act_ready() returns (also after an abort, so that every armed stage completes).
     bool waited = false;
     int npend = 0;
     Ring rg(S);
@@ -257,7 +303,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
         }
         if (leader) {
           if (g < 16) DPTQ_TRACE_POINT(tr, 8 + g);
-          mbar_arrive_expect_tx(&full[s], tx);
+          mbar_arrive_expect_tx(&full[s], w_bytes);
           bulk_g2s(sm.wpack(s), wsrc, w_bytes, &full[s], pol_w);
           if (waited)
             issue_act(s, asrc);
@@ -266,7 +312,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
           if (g < 16) DPTQ_TRACE_POINT(tr, 24 + g);
         }
         if (!waited && ++npend == S) {
-          pdl_wait();
+          if (!act_ready()) ok = false;
           waited = true;
           __syncwarp();
           if (leader)
@@ -274,12 +320,16 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
           npend = 0;
         }
         __syncwarp();
+        if (!ok) {
+          ++g;   // this stage is armed: the drain below must see it
+          break;
+        }
       }
     }
     // Stages armed before the wait for the previous kernel still expect their
     // activation bytes (also after an abort, so that the drain below completes).
     if (!waited) {
-      pdl_wait();
+      act_ready();
       __syncwarp();
       if (leader)
         for (int i = 0; i < npend; ++i) issue_act(i, pend_src[i]);
@@ -288,8 +338,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
     // Do not leave the CTA while copies into its shared memory may be in flight.
     if (*abort_flag) {
       volatile int no_abort = 0;
-      for (int gg = (g > S ? g - S : 0); gg < g; ++gg)
+      for (int gg = (g > S ? g - S : 0); gg < g; ++gg) {
         mbar_wait_warp(&full[gg % S], (gg / S) & 1, &no_abort, a.err, kDevTimeoutDrain);
+        mbar_wait_warp(&afull[gg % S], (gg / S) & 1, &no_abort, a.err, kDevTimeoutDrain);
+      }
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
@@ -321,7 +373,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
       bool ok = true;
       for (int it = un.i0; it < un.i1; ++it, rg.next(), rc.next()) {
         const int s = rg.s, c = rc.s;
-        if (!mbar_wait_warp(&cfull[c], rc.ph, abort_flag, a.err, kDevTimeoutConv)) {
+        if (!mbar_wait_warp(&afull[s], rg.ph, abort_flag, a.err, kDevTimeoutFull) ||
+            !mbar_wait_warp(&cfull[c], rc.ph, abort_flag, a.err, kDevTimeoutConv)) {
           ok = false;
           break;
         }
@@ -376,6 +429,25 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
   } else if (warp < kEpiWarp0) {
     // ------------------------------------------------------------ converters
     const int ctid = threadIdx.x - kConvWarp0 * 32;   // 0..255
+    if constexpr (FUSED) {
+      // Rotate + quantize token rows c, c + G, ... into the activation planes and
+      // scales, then publish them.  The 8 converter warps meet at named barrier 1.
+      pdl_wait();   // the rows come from the previous kernel
+      if (ctid == 0) DPTQ_TRACE_POINT(tr, 125);
+      const auto csync = [] { asm volatile("bar.sync 1, %0;" ::"n"(kConvThreads) : "memory"); };
+      int nrows = 0;
+      for (int row = blockIdx.x; row < a.M_pad; row += gridDim.x) {
+        if (nrows) csync();   // the previous row's readers are done with the scratch
+        rotate_quant_row<kRQAct>(a.rq, row, rot_smem, rot_red, ctid, csync);
+        ++nrows;
+      }
+      if (ctid == 0) DPTQ_TRACE_POINT(tr, 126);
+      if (nrows) {
+        csync();   // every converter thread's code and scale stores precede the release
+        if (ctid == 0) release_add_gpu(a.gsync, (uint32_t)nrows);
+      }
+      if (ctid == 0) DPTQ_TRACE_POINT(tr, 127);
+    }
     Ring rg(S), rc(CS);
     int cvt_done = 0;
     while (iter.next(un)) {
@@ -450,6 +522,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
   } else {
     // ------------------------------------------------------------ epilogue
     pdl_wait();   // scales come from the previous kernel; `out` may still be read by it
+    bool epi_ok = true;
+    if constexpr (FUSED) epi_ok = mbar_wait(aready, 0, abort_flag, a.err, kDevTimeoutGrid);
     const float* __restrict__ sa_g = a.sa;
     const float* __restrict__ sw_g = a.sw;
     __half* __restrict__ out_g = a.out;
@@ -470,7 +544,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
     };
     int sa_mt = -1;   // token tile whose activation scales sit in sa_sh
     int u = 0;
-    while (iter.next(un)) {
+    while (epi_ok && iter.next(un)) {
       const int b = a.nbuf == 2 ? (u & 1) : 0;
       const uint32_t tpar = (a.nbuf == 2 ? (u >> 1) : u) & 1;
       const int nt = un.tile / a.m_tiles;
@@ -671,6 +745,17 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
     tc_fence_after();
     tmem_dealloc(tmem_base, a.tmem_cols);
   }
+  if constexpr (FUSED) {
+    // Every producer has passed its wait on the row counter: the last CTA out resets
+    // both counters for the next launch (which reads them only after this grid ends).
+    if (threadIdx.x == 0) {
+      const uint32_t prev = atom_add_acq_rel_gpu(a.gsync + 1, 1u);
+      if (prev == gridDim.x - 1) {
+        a.gsync[0] = 0u;
+        a.gsync[1] = 0u;
+      }
+    }
+  }
   if (threadIdx.x == 0) DPTQ_TRACE_POINT(tr, 120);
 }
 
@@ -693,7 +778,7 @@ static int smem_for(int nt, int kps, int stages, int planes, int conv_slots) {
   return 1024 + conv_slots * kps * kConvBytes + stages * kps * (planes * nt * 128 + kWTileBytes) + kBarrierBytes;
 }
 
-bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan) {
+bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan, int rot_smem) {
   GemmArgs& a = plan.args;
   const int KB = K_pad / kKBlock;
   const int planes = bits == 8 ? 2 : 1;
@@ -728,9 +813,14 @@ bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan) {
   if (!a_tmem)
     while (conv_slots > 2 && smem_for(nt, kps, 4, planes, conv_slots) > kSmemLimit) --conv_slots;
   const int smem_conv = a_tmem ? 0 : conv_slots;
+  // A fused launch needs two-block stages (weights widened into TMEM) and room for one
+  // row's rotation scratch next to at least 3 stages.
+  const bool fused = rot_smem > 0;
+  if (fused && kps != 2) return false;
+  auto smem_total = [&](int st) { return smem_for(nt, kps, st, planes, smem_conv) + (fused ? rot_smem : 0); };
   int stages = kMaxStages;
-  while (stages > 2 && smem_for(nt, kps, stages, planes, smem_conv) > kSmemLimit) --stages;
-  if (smem_for(nt, kps, stages, planes, smem_conv) > kSmemLimit) return false;
+  while (stages > 2 && smem_total(stages) > kSmemLimit) --stages;
+  if (smem_total(stages) > kSmemLimit || (fused && stages < 3)) return false;
   const int a_cols = a_tmem ? conv_slots * kps * 32 : 0;
   const int nbuf = 2 * nt * segs + a_cols <= 512 ? 2 : 1;
   if (nbuf * nt * segs + a_cols > 512) return false;
@@ -749,11 +839,12 @@ bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan) {
   long long dp = 0;
   if (tiles >= 2LL * G) dp = (tiles / G - 1) * G;
 
+  plan.fused = fused;
   plan.nt = nt;
   plan.kps = kps;
   plan.M_pad = M_pad;
   plan.grid = G;
-  plan.smem_bytes = smem_for(nt, kps, stages, planes, smem_conv);
+  plan.smem_bytes = smem_total(stages);
   a.M = M;
   a.N = N;
   a.M_pad = M_pad;
@@ -774,13 +865,15 @@ bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan) {
   if ((long long)a.sk_iters * G + G >= (1LL << 32) || tiles >= (1LL << 31)) return false;
   a.tmem_cols = cols;
   a.out_vec = 0;
+  a.rq = RQArgs{};
+  a.gsync = nullptr;
   return true;
 }
 
-template <int NT, int KPS>
+template <int NT, int KPS, bool FUSED = false>
 static cudaError_t launch_nt(const GemmPlan& plan, cudaStream_t s, bool pdl) {
-  cudaError_t e =
-      cudaFuncSetAttribute(qgemm_kernel<NT, KPS>, cudaFuncAttributeMaxDynamicSharedMemorySize, plan.smem_bytes);
+  cudaError_t e = cudaFuncSetAttribute(qgemm_kernel<NT, KPS, FUSED>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       plan.smem_bytes);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)plan.grid);
@@ -792,10 +885,18 @@ static cudaError_t launch_nt(const GemmPlan& plan, cudaStream_t s, bool pdl) {
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = (pdl && pdl_allowed()) ? 1 : 0;
-  return cudaLaunchKernelEx(&cfg, qgemm_kernel<NT, KPS>, plan.args);
+  return cudaLaunchKernelEx(&cfg, qgemm_kernel<NT, KPS, FUSED>, plan.args);
 }
 
 cudaError_t launch_gemm(const GemmPlan& plan, cudaStream_t s, bool pdl) {
+  if (plan.fused) {
+    switch (plan.nt) {
+      case 16: return launch_nt<16, 2, true>(plan, s, pdl);
+      case 32: return launch_nt<32, 2, true>(plan, s, pdl);
+      case 64: return launch_nt<64, 2, true>(plan, s, pdl);
+      default: return cudaErrorInvalidValue;
+    }
+  }
   if (plan.kps == 2) {
     switch (plan.nt) {
       case 16: return launch_nt<16, 2>(plan, s, pdl);
@@ -817,7 +918,7 @@ cudaError_t launch_gemm(const GemmPlan& plan, cudaStream_t s, bool pdl) {
 }  // namespace dptq
 
 #ifdef DPTQ_TRACE
-// Trace builds only: set (or clear with NULL) the device buffer of 128 stamps per CTA.
+// Trace builds only: set (or clear with NULL) the device buffer of 256 stamps per CTA.
 extern "C" int dptq_trace_set(void* dev_buffer) {
   return (int)cudaMemcpyToSymbol(dptq::g_dptq_trace, &dev_buffer, sizeof(dev_buffer));
 }

@@ -248,6 +248,28 @@ def test_qlinear_unaligned_output(dp, M, N, K, B):
     layer.close()
 
 
+@pytest.mark.parametrize("M,N,K,B", [(64, 128, 256, 256), (16, 512, 256, 256), (5, 4096, 4096, 4096),
+                                     (32, 4096, 11008, 256), (33, 1024, 2048, 512), (1, 22016, 4096, 4096)])
+def test_fused_qlinear_equals_two_launches(dp, M, N, K, B):
+    """dptq_qlinear (one launch for small M: the GEMM kernel rotates and quantizes the rows
+    itself) gives the same bits as the rotate-quantize launch followed by the GEMM launch.
+    (64, 128, 256): one CTA quantizes all 64 rows; (16, 512, 256): 4 CTAs, 4 rows each."""
+    wl = inputs.llama2_7b_decode()
+    x = torch.from_numpy(inputs.activations(wl, M, K)).to(DEV)
+    W = inputs.weights(N, K, layer=7, proj=1)
+    layer = dp.dptq_pack_weights(torch.from_numpy(W).to(DEV), B)
+    for bits in (4, 8):
+        fused = torch.empty((M, N), dtype=torch.float16, device=DEV)
+        two = torch.empty((M, N), dtype=torch.float16, device=DEV)
+        for _ in range(3):   # repeated launches reuse the grid counters
+            dp.dptq_qlinear(layer, x, bits, fused)
+        dp.dptq_qlinear_quantize(layer, x, bits)
+        dp.dptq_qlinear_gemm(layer, M, bits, two)
+        torch.cuda.synchronize()
+        assert torch.equal(fused.view(torch.int16), two.view(torch.int16)), (M, N, K, bits)
+    layer.close()
+
+
 def test_qlinear_m_zero_is_noop(dp):
     W = inputs.weights(128, 256)
     layer = dp.dptq_pack_weights(torch.from_numpy(W).to(DEV), 256)
