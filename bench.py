@@ -346,6 +346,105 @@ def e2e_measure(stack, g, stream, steps, world):
     return max(e0.elapsed_time(e1) / 1e3, 0.0) / steps, wall / steps
 
 
+# ------------------------------------------------------------------------------ per-shape kernels
+L2_BYTES = 129 * 2 ** 20
+
+
+def shape_cases():
+    """(label, M, N, K, had_block, bits): the LLaMA-2-7B decode projections and the
+    LLaMA-3-8B prefill ones (gate|up as one concatenated N)."""
+    d = [("7b qkv", 12288, 4096, 4096), ("7b o", 4096, 4096, 4096), ("7b gate|up", 22016, 4096, 4096),
+         ("7b down", 4096, 11008, 256)]
+    out = [(f"{n} decode", 32, N, K, B, 4) for n, N, K, B in d]
+    out += [("7b gate|up decode", 32, 22016, 4096, 4096, 8), ("7b gate|up decode", 1, 22016, 4096, 4096, 4),
+            ("7b gate|up decode", 8, 22016, 4096, 4096, 4)]
+    out += [("8b q prefill", 2048, 4096, 4096, 2048, 4), ("8b gate|up prefill", 2048, 28672, 4096, 2048, 4),
+            ("8b down prefill", 2048, 4096, 14336, 2048, 4)]
+    return out
+
+
+def run_shapes(args):
+    """Times one launch of each shape (CUDA events over graph replays of 40 launches) with
+    as many weight copies as make the rotation through them at least twice the L2, so
+    every launch streams its weights from HBM."""
+    import math
+    import torch
+    from paper_2606_12487_gb300 import dptq, inputs
+    dptq.load()
+    dev = torch.device("cuda")
+    dptq.dptq_reserve(2048, 14336, 0)
+    peaks = {}
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            peaks = json.load(f)
+    except OSError:
+        pass
+    hbm = float(peaks.get("hbm_gbs", 6800.0))
+    fp8 = 2.0 * float(peaks.get("bf16_tflops", 1900.0))
+    stream = torch.cuda.Stream(device=dev)
+    reps = 40
+
+    def t_graph(fns):
+        with torch.cuda.stream(stream):
+            for f in fns[:3]:
+                f()
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for i in range(reps):
+                fns[i % len(fns)]()
+        for _ in range(2):
+            g.replay()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            g.replay()
+            e1.record(stream)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) * 1e3 / reps
+
+    rows = []
+    for label, M, N, K, B, bits in shape_cases():
+        wbytes = N * K // 2
+        copies = max(1, min(64, math.ceil(2 * L2_BYTES / wbytes)))
+        W = inputs.torch_weights(N, K, 0, 0, dev)
+        hs = [dptq.dptq_pack_weights(W, B) for _ in range(copies)]
+        del W
+        x = torch.from_numpy(inputs.activations(inputs.llama2_7b_decode(), M, K)).to(dev)
+        out = torch.empty((M, N), dtype=torch.float16, device=dev)
+        s_ = stream
+        t_q = t_graph([lambda h=h: dptq.dptq_qlinear_quantize(h, x, bits, stream=s_) for h in hs[:1]])
+        with torch.cuda.stream(stream):
+            dptq.dptq_qlinear_quantize(hs[0], x, bits, stream=s_)
+        t_g = t_graph([lambda h=h: dptq.dptq_qlinear_gemm(h, M, bits, out, stream=s_) for h in hs])
+        t_l = t_graph([lambda h=h: dptq.dptq_qlinear(h, x, bits, out, stream=s_) for h in hs])
+        gemm_b = wbytes + 4 * N + M * K * bits // 8 + 4 * M + 2 * M * N
+        ql_b = wbytes + 4 * N + 2 * M * K + 2 * M * N
+        ops = 2 * M * N * K
+        r = {"shape": label, "M": M, "N": N, "K": K, "had_block": B, "bits": bits, "weight_copies": copies,
+             "quantize_us": t_q, "gemm_us": t_g, "qlinear_us": t_l,
+             "gemm_gbs": gemm_b / t_g / 1e3, "qlinear_gbs": ql_b / t_l / 1e3,
+             "gemm_tops": ops / t_g / 1e6, "qlinear_tops": ops / t_l / 1e6}
+        if M <= 64:
+            r["roofline"] = {"bound": "hbm", "peak_gbs": hbm, "gemm_frac": r["gemm_gbs"] / hbm,
+                             "qlinear_frac": r["qlinear_gbs"] / hbm}
+        else:
+            r["roofline"] = {"bound": "tensor", "peak_tflops": fp8, "peak_note": "2 x bf16 burst measured (fp8 nominal ratio)",
+                             "gemm_frac": r["gemm_tops"] / fp8, "qlinear_frac": r["qlinear_tops"] / fp8}
+        rows.append(r)
+        print(f"[shapes] {label} M={M} A{bits}: quantize {t_q:.1f} us, gemm {t_g:.1f} us, qlinear {t_l:.1f} us",
+              file=sys.stderr, flush=True)
+        for h in hs:
+            h.close()
+        del hs
+        torch.cuda.synchronize()
+    dptq.dptq_last_device_error()
+    print(json.dumps({"mode": "shapes", "timing": "CUDA events over graph replays, weights rotated through "
+                                                  ">= 2x L2 of copies", "shapes": rows}), flush=True)
+    return 0
+
+
 # ------------------------------------------------------------------------------ oracle timing
 def oracle_sample_times(wl, budget_s: float, tokens: int = 1):
     """Time the oracle's online path (rotate + quantize, int GEMM, epilogue) per layer
@@ -466,11 +565,15 @@ def main(argv=None):
                          "split: rotate-quantize launch, then GEMM launch")
     ap.add_argument("--layers", type=int, default=0,
                     help="run only the first L layers (small cases for profiler captures; 0 = all)")
+    ap.add_argument("--shapes", action="store_true",
+                    help="time each decode / prefill projection shape alone and print one JSON line of them")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         args.warmup = 3
     if args.impl == "reference":
         return run_reference(args)
+    if args.shapes:
+        return run_shapes(args)
 
     import torch
     rank, world, local = dist_env()

@@ -98,9 +98,14 @@ dptq_status dptq_rotate_act(const void* x_fp16, int M, int K, int had_block, flo
 /* The quantized linear layer: out = fp16( Q(x R) (W R)^T scaled ), i.e. rotate and
  * quantize x with `bits` (4 or 8, the layer's mask entry), multiply by the packed
  * int4 weights of `h` with exact int32 accumulation, apply s_a[m] * s_w[n].
- * x_fp16: device [M][K]; out_fp16: device [M][N] (written).  Asynchronous.
+ * x_fp16: device [M][K]; out_fp16: device [M][N] (written; any alignment, a 16-byte
+ * aligned pointer is written 8 bytes at a time).  Asynchronous.
  * Uses the library's per-device scratch (grown on demand; call dptq_reserve before
- * capturing into a CUDA graph so that no allocation happens during capture). */
+ * capturing into a CUDA graph so that no allocation happens during capture).
+ * For token tiles of up to 64 rows (M <= 64) whose rotation fits next to the GEMM's
+ * pipeline in one CTA's shared memory, rotation, quantization and GEMM run as ONE
+ * kernel launch (the environment variable DPTQ_FUSED=0 selects the two-launch
+ * sequence of dptq_qlinear_quantize + dptq_qlinear_gemm); both give the same bits. */
 dptq_status dptq_qlinear(dptq_handle h, const void* x_fp16, int M, int bits, void* out_fp16,
                          void* stream);
 

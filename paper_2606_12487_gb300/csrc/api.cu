@@ -113,6 +113,9 @@ bool capturing(cudaStream_t s) {
 }
 
 constexpr int kMaxNT = 256;
+// Rows of up to 4 chunks of 4096 take the fused launch (its rotation runs each row's
+// butterflies twice when the row has more than one chunk).
+constexpr int kFusedMaxKPad = 16384;
 
 // Make sure the device's scratch holds `act_bytes` of activation planes and `sa_count`
 // scales.  Growth allocates, so it is refused while `s` is being captured.
@@ -339,9 +342,8 @@ dptq_status dptq_qlinear(dptq_handle h, const void* x_fp16, int M, int bits, voi
   if (!x_fp16 || !out_fp16) return fail(DPTQ_ERR_INVALID_ARG, "null pointer");
   // Small M: one launch that rotates and quantizes the rows and runs the GEMM.
   GemmPlan fp;
-  if (fused_allowed() &&
-      plan_gemm(M, h->N, h->K_pad, bits, sc->num_sms, fp, (int)rotate_quant_smem(h->K, 0)) &&
-      fp.M_pad == plan.M_pad) {
+  if (fused_allowed() && h->K_pad <= kFusedMaxKPad &&
+      plan_gemm(M, h->N, h->K_pad, bits, sc->num_sms, fp, kRQPartSmemBytes) && fp.M_pad == plan.M_pad) {
     int nfull, tail, log2B;
     if ((st = check_shape(h->K, h->had_block, nfull, tail, log2B)) != DPTQ_OK) return st;
     fp.args.rq = make_rq(x_fp16, M, fp.M_pad, h->K, h->KB, h->had_block, nfull, tail, log2B, bits, sc->sa, sc->act);

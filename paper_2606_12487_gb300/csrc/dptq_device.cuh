@@ -29,7 +29,14 @@ __device__ __forceinline__ unsigned long long trace_now() {
     if (buf) (buf)[blockIdx.x * 256 + (slot)] = (unsigned long long)(v); \
   } while (0)
 #define DPTQ_TRACE_BUF() ::dptq::g_dptq_trace
+#define DPTQ_TRACE_CLOCK(buf, slot) \
+  do {                              \
+    if (buf) (buf)[blockIdx.x * 256 + (slot)] = (unsigned long long)clock64(); \
+  } while (0)
 #else
+#define DPTQ_TRACE_CLOCK(buf, slot) \
+  do {                              \
+  } while (0)
 #define DPTQ_TRACE_POINT(buf, slot) \
   do {                              \
   } while (0)

@@ -55,6 +55,10 @@ struct RQArgs {
 };
 
 cudaError_t launch_rotate_quant(RQMode mode, const RQArgs& a, cudaStream_t s, bool pdl);
+// Shared memory of one row part in the fused decode launch: the padded int64 transpose
+// chunk (4096 + 256 values), two planes of staged codes (4096 bytes each) and 16 warp
+// maxima.
+constexpr int kRQPartSmemBytes = (4096 + 256) * 8 + 2 * 4096 + 16 * 8;
 size_t rotate_quant_smem(int K, int chunk);
 // Shared-memory budget of one CTA (227 KB opt-in).
 constexpr size_t kSmemPerBlock = 232448;
@@ -96,6 +100,8 @@ struct GemmArgs {
   // (written to `act` / `sa` by the converter warps of CTAs 0, 1, ...) and the two grid
   // counters [rows ready, CTAs done] that order it before the GEMM (zero between launches).
   RQArgs rq;
+  int rq_np;           // parts per token row (1, 2 or 4): work item = row * rq_np + part
+  int rq_items;        // M_pad * rq_np: the value the rows-ready counter reaches
   uint32_t* gsync;
 };
 

@@ -183,7 +183,6 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
   volatile int* flags = reinterpret_cast<volatile int*>(tmem_base_sh + 2);   // epilogue: 2 units x 2
   float* sa_sh = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + 512);   // token scales (NT <= 64)
   __half* xpose = reinterpret_cast<__half*>(reinterpret_cast<uint8_t*>(bars) + 1024);  // 4 x [4 tokens][32 ch]
-  float* rot_red = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + 768);   // fused: 8 warp maxima
   unsigned char* rot_smem = reinterpret_cast<unsigned char*>(bars) + kBarrierBytes;    // fused: one row's scratch
   const uint8_t** pend_src = reinterpret_cast<const uint8_t**>(tmem_base_sh + 8);   // producer's pending list
 
@@ -258,7 +257,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
         while (true) {
           int st = 0;
           if (lane == 0) {
-            if (ld_acquire_gpu(a.gsync) >= (uint32_t)a.M_pad)
+            if (ld_acquire_gpu(a.gsync) >= (uint32_t)a.rq_items)
               st = 1;
             else if (*abort_flag)
               st = 2;
@@ -430,21 +429,28 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
     // ------------------------------------------------------------ converters
     const int ctid = threadIdx.x - kConvWarp0 * 32;   // 0..255
     if constexpr (FUSED) {
-      // Rotate + quantize token rows c, c + G, ... into the activation planes and
-      // scales, then publish them.  The 8 converter warps meet at named barrier 1.
+      // Rotate + quantize work items c, c + G, ... (item = row * rq_np + part) into the
+      // activation planes and scales, then publish them.  The 8 converter warps meet
+      // at named barrier 1.
       pdl_wait();   // the rows come from the previous kernel
-      if (ctid == 0) DPTQ_TRACE_POINT(tr, 125);
-      const auto csync = [] { asm volatile("bar.sync 1, %0;" ::"n"(kConvThreads) : "memory"); };
-      int nrows = 0;
-      for (int row = blockIdx.x; row < a.M_pad; row += gridDim.x) {
-        if (nrows) csync();   // the previous row's readers are done with the scratch
-        rotate_quant_row<kRQAct>(a.rq, row, rot_smem, rot_red, ctid, csync);
-        ++nrows;
+      if (ctid == 0) {
+        DPTQ_TRACE_POINT(tr, 125);
+        DPTQ_TRACE_CLOCK(tr, 160);
       }
-      if (ctid == 0) DPTQ_TRACE_POINT(tr, 126);
-      if (nrows) {
+      const auto csync = [] { asm volatile("bar.sync 1, %0;" ::"n"(kConvThreads) : "memory"); };
+      int nitems = 0;
+      for (int item = blockIdx.x; item < a.rq_items; item += gridDim.x) {
+        if (nitems) csync();   // the previous item's readers are done with the scratch
+        rotate_quant_row_part(a.rq, item / a.rq_np, item % a.rq_np, a.rq_np, rot_smem, ctid, csync);
+        ++nitems;
+      }
+      if (ctid == 0) {
+        DPTQ_TRACE_POINT(tr, 126);
+        DPTQ_TRACE_CLOCK(tr, 161);
+      }
+      if (nitems) {
         csync();   // every converter thread's code and scale stores precede the release
-        if (ctid == 0) release_add_gpu(a.gsync, (uint32_t)nrows);
+        if (ctid == 0) release_add_gpu(a.gsync, (uint32_t)nitems);
       }
       if (ctid == 0) DPTQ_TRACE_POINT(tr, 127);
     }
@@ -867,6 +873,12 @@ bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan, i
   a.out_vec = 0;
   a.rq = RQArgs{};
   a.gsync = nullptr;
+  // Fused: up to 4 CTAs share each token row (each converts and writes a quarter of it),
+  // as long as every part has a CTA of its own.
+  int np = fused ? 4 : 1;
+  while (np > 1 && (long long)M_pad * np > G) np >>= 1;
+  a.rq_np = np;
+  a.rq_items = fused ? M_pad * np : 0;
   return true;
 }
 

@@ -65,6 +65,35 @@ __device__ __forceinline__ int quantize(float y, float s, float r, int qmin, int
   return (int)quant_code(y, s, r, (float)qmin, (float)qmax);
 }
 
+// The same for four values at once, by a whole warp: the reciprocal products for all
+// four, then (only if some lane of the warp has a value near a half-integer) the IEEE
+// quotients of those values, so that the common path carries no division code.
+__device__ __forceinline__ void quant_code4(const float (&y)[4], float s, float r, float qmin, float qmax,
+                                            float (&c)[4]) {
+  uint32_t nearm = 0;
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const float t = __fmul_rn(y[j], r);
+    c[j] = rintf(t);
+    nearm |= (fabsf(__fsub_rn(t, c[j])) >= 0.5f - 0x1p-15f) ? (1u << j) : 0u;
+  }
+  if (__any_sync(__activemask(), nearm != 0u)) {
+#pragma unroll 1
+    for (int j = 0; j < 4; ++j) {
+      if ((nearm >> j) & 1u) {
+        const float yj = j == 0 ? y[0] : j == 1 ? y[1] : j == 2 ? y[2] : y[3];
+        const float q = rintf(__fdiv_rn(yj, s));
+        if (j == 0) c[0] = q;
+        if (j == 1) c[1] = q;
+        if (j == 2) c[2] = q;
+        if (j == 3) c[3] = q;
+      }
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < 4; ++j) c[j] = __fadd_rn(fminf(fmaxf(c[j], qmin), qmax), 0.0f);   // -0 -> +0
+}
+
 // Two small integers (exact in E4M3) to FP8 E4M3 bytes: lo in bits 0-7, hi in 8-15.
 __device__ __forceinline__ uint32_t e4m3x2(float lo, float hi) {
   uint16_t d;
@@ -369,10 +398,8 @@ __device__ __forceinline__ void rotate_quant_row(const RQArgs& a, int row, unsig
         float c[4] = {0.f, 0.f, 0.f, 0.f};
         if (nz && k < K) {   // K % 32 == 0: the four codes are all inside K or all padding
           const float4 y4 = *reinterpret_cast<const float4*>(sy + k);
-          c[0] = quant_code(y4.x, s, rs, qminf, qmaxf);
-          c[1] = quant_code(y4.y, s, rs, qminf, qmaxf);
-          c[2] = quant_code(y4.z, s, rs, qminf, qmaxf);
-          c[3] = quant_code(y4.w, s, rs, qminf, qmaxf);
+          const float yv[4] = {y4.x, y4.y, y4.z, y4.w};
+          quant_code4(yv, s, rs, qminf, qmaxf, c);
         }
         const int kb = k >> 7, j = (k >> 4) & 7;
         const size_t off = ((size_t)kb * a.rows_out + row) * 128 + ((j ^ (row & 7)) << 4) + (k & 15);
@@ -425,6 +452,329 @@ __device__ __forceinline__ void rotate_quant_row(const RQArgs& a, int row, unsig
     }
   }
 #undef RQ_TRACE
+}
+
+// ---------------------------------------------------------------- fused decode launch
+// Element index of value e of thread t in the layout the butterflies of a chunk end in:
+// 0 = round A only (blocks of at most 16), 1 = rounds A and B (at most 256), 2 = all.
+__device__ __forceinline__ int rq_pos(int layout, int t, int e) {
+  return layout == 2 ? 256 * e + t : layout == 1 ? 256 * (t >> 4) + 16 * e + (t & 15) : 16 * t + e;
+}
+
+// The exact butterflies of one chunk (elements c0 .. c0 + len - 1 of the row at `src`),
+// the same arithmetic as rotate_quant_row; returns the layout f[] ends in.
+template <class Sync>
+__device__ __forceinline__ int rq_chunk(const RQArgs& a, const uint4* src, int c0, int len, int tail_start,
+                                        long long (&f)[16], long long* sx, int tid, Sync sync) {
+  unsigned long long* const tr = DPTQ_TRACE_BUF();
+  (void)tr;
+#define RQC_T(slot) \
+  do {              \
+    if (tid == 0 && c0 == 0) DPTQ_TRACE_CLOCK(tr, slot); \
+  } while (0)
+  RQC_T(170);
+  auto lg = [&](int i) { return (c0 + i < tail_start) ? a.log2B : a.log2T; };
+  auto bfly = [&](int h) {
+#pragma unroll
+    for (int e = 0; e < 16; ++e)
+      if ((e & h) == 0) {
+        const long long p = f[e], q = f[e + h];
+        f[e] = p + q;
+        f[e + h] = p - q;
+      }
+  };
+  const int i0 = tid * 16;
+  if (i0 < len) {
+    const uint4 u0 = src[(c0 + i0) / 8];
+    const uint4 u1 = src[(c0 + i0) / 8 + 1];
+    const uint32_t w[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      f[2 * k] = half_to_fixed(w[k] & 0xFFFFu);
+      f[2 * k + 1] = half_to_fixed(w[k] >> 16);
+    }
+  } else {
+#pragma unroll
+    for (int k = 0; k < 16; ++k) f[k] = 0;
+  }
+  if (tid == 0 && c0 == 0) { volatile long long sink = f[0] ^ f[15]; (void)sink; }
+  RQC_T(171);
+  {
+    const int L = lg(i0 < len ? i0 : 0);
+    if (L >= 4) {
+      bfly(1);
+      bfly(2);
+      bfly(4);
+      bfly(8);
+    } else {
+#pragma unroll
+      for (int bit = 0; bit < 4; ++bit)
+        if (bit < L) bfly(1 << bit);
+    }
+  }
+  if (tid == 0 && c0 == 0) { volatile long long sink = f[0] ^ f[15]; (void)sink; }
+  RQC_T(172);
+  const int maxlg = (c0 + len > tail_start) ? max(a.log2B, a.log2T) : a.log2B;
+  if (maxlg <= 4) return 0;
+  sync();   // the previous readers of sx are done
+#pragma unroll
+  for (int e = 0; e < 16; ++e) sx[pad_idx(i0 + e)] = f[e];
+  sync();
+  const int iB = 256 * (tid >> 4) + (tid & 15);
+#pragma unroll
+  for (int e = 0; e < 16; ++e) f[e] = sx[pad_idx(iB + 16 * e)];
+  if (tid == 0 && c0 == 0) { volatile long long sink = f[0] ^ f[15]; (void)sink; }
+  RQC_T(173);
+  {
+    const int L = lg(iB);
+    if (L >= 8) {
+      bfly(1);
+      bfly(2);
+      bfly(4);
+      bfly(8);
+    } else {
+#pragma unroll
+      for (int bit = 4; bit < 8; ++bit)
+        if (bit < L) bfly(1 << (bit - 4));
+    }
+  }
+  if (tid == 0 && c0 == 0) { volatile long long sink = f[0] ^ f[15]; (void)sink; }
+  RQC_T(174);
+  if (maxlg <= 8) return 1;
+#pragma unroll
+  for (int e = 0; e < 16; ++e) sx[pad_idx(iB + 16 * e)] = f[e];
+  sync();
+#pragma unroll
+  for (int e = 0; e < 16; ++e) f[e] = sx[pad_idx(256 * e + tid)];
+  if (tid == 0 && c0 == 0) { volatile long long sink = f[0] ^ f[15]; (void)sink; }
+  RQC_T(175);
+  if (c0 + len <= tail_start && a.log2B == 12) {
+    bfly(1);
+    bfly(2);
+    bfly(4);
+    bfly(8);
+  } else if (c0 + len <= tail_start) {
+#pragma unroll
+    for (int bit = 8; bit < 12; ++bit)
+      if (bit < a.log2B) bfly(1 << (bit - 8));
+  } else {
+#pragma unroll
+    for (int bit = 8; bit < 12; ++bit) {
+      const int h = 1 << (bit - 8);
+#pragma unroll
+      for (int e = 0; e < 16; ++e)
+        if ((e & h) == 0 && bit < lg(256 * e + tid)) {
+          const long long p = f[e], q = f[e + h];
+          f[e] = p + q;
+          f[e + h] = p - q;
+        }
+    }
+  }
+  if (tid == 0 && c0 == 0) { volatile long long sink = f[0] ^ f[15]; (void)sink; }
+  RQC_T(176);
+#undef RQC_T
+  return 2;
+}
+
+__device__ __forceinline__ uint32_t e4m3_byte(float v) { return e4m3x2(v, 0.f) & 0xFFu; }
+
+static_assert(kRQPartSmemBytes == kChunkPadded * 8 + 2 * kChunk + 16 * 8, "part scratch layout");
+
+// The share `part` of `np` (1, 2 or 4) of one row in the fused decode launch, writing
+// the GEMM operand planes (kRQAct layout) and, for part 0, the row's scale.  Every part
+// runs the row's butterflies (cheap), and takes the absmax from the largest |S| of each
+// block size: the conversion to fp32 is odd and monotone in S, so max|y| is the
+// conversion of max|S|.  It then converts, quantizes and writes only the values whose
+// index e (in the final layout) lies in [16 part / np, 16 (part + 1) / np), staging the
+// codes in shared memory for coalesced 32-bit stores.  Rows of more than one chunk run
+// the butterflies twice (the values are not kept).  Codes and scales equal those of
+// rotate_quant_row<kRQAct>.  smem: kRQPartSmemBytes, 16-byte aligned; 256 threads meet
+// at sync(); the caller synchronizes before reusing smem for another row.
+template <class Sync>
+__device__ __forceinline__ void rotate_quant_row_part(const RQArgs& a, int row, int part, int np,
+                                                      unsigned char* smem, int tid, Sync sync) {
+  long long* sx = reinterpret_cast<long long*>(smem);
+  uint8_t* cst = smem + (size_t)kChunkPadded * 8;                 // [2][kChunk] staged E4M3 codes
+  long long* red = reinterpret_cast<long long*>(cst + 2 * kChunk);   // [16] warp maxima
+  unsigned long long* const tr = DPTQ_TRACE_BUF();
+  (void)tr;
+  const int K = a.K;
+  const int K_pad = a.KB * 128;
+  const bool live = row < a.rows_in;
+  const int tail_start = a.nfull << a.log2B;
+  const int bits = a.bits;
+  const int qmax = (1 << (bits - 1)) - 1;
+  const float qmaxf = (float)qmax, qminf = (float)(-(1 << (bits - 1)));
+  uint8_t* act = static_cast<uint8_t*>(a.out);
+  const size_t plane_stride = (size_t)a.KB * a.rows_out * 128;
+  auto store4 = [&](int k, uint32_t w0, uint32_t w1) {   // codes k .. k + 3 (k % 4 == 0)
+    const int kb = k >> 7, j = (k >> 4) & 7;
+    const size_t off = ((size_t)kb * a.rows_out + row) * 128 + ((j ^ (row & 7)) << 4) + (k & 15);
+    *reinterpret_cast<uint32_t*>(act + off) = w0;
+    if (bits == 8) *reinterpret_cast<uint32_t*>(act + plane_stride + off) = w1;
+  };
+
+  if (!live) {   // padding row: zero codes (words split evenly over the parts) and scale
+    const int W = K_pad / 4;
+    for (int w = W * part / np + tid; w < W * (part + 1) / np; w += kRQThreads) store4(4 * w, 0u, 0u);
+    if (part == 0 && tid == 0 && a.scales != nullptr) a.scales[row] = 0.f;
+    return;
+  }
+
+  const uint4* src = reinterpret_cast<const uint4*>(a.x + (size_t)row * K);
+  long long f[16];
+  int L0 = 0;
+  // With 4 parts and at most 3 chunks, each chunk's 4 values of this part are converted
+  // to fp32 in pass 1 (the conversion does not depend on the scale) and stay in
+  // registers (kept[chunk]) for pass 2; otherwise pass 2 repeats the butterflies.
+  const bool keep = np == 4 && K <= 3 * kChunk;
+  float kept[3][4];
+  int kept_L[3] = {0, 0, 0};
+  // ---- pass 1: butterflies, largest |S| per block size
+  long long mB = 0, mT = 0;
+  for (int c0 = 0; c0 < K; c0 += kChunk) {
+    const int len = min(kChunk, K - c0);
+    const int L = rq_chunk(a, src, c0, len, tail_start, f, sx, tid, sync);
+    L0 = L;
+    if (keep) {
+      long long w[4];
+      switch (part) {
+        case 0: w[0] = f[0]; w[1] = f[1]; w[2] = f[2]; w[3] = f[3]; break;
+        case 1: w[0] = f[4]; w[1] = f[5]; w[2] = f[6]; w[3] = f[7]; break;
+        case 2: w[0] = f[8]; w[1] = f[9]; w[2] = f[10]; w[3] = f[11]; break;
+        default: w[0] = f[12]; w[1] = f[13]; w[2] = f[14]; w[3] = f[15]; break;
+      }
+      float v[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int i = rq_pos(L, tid, 4 * part + j);
+        v[j] = i < len ? fixed_to_rotated(w[j], (c0 + i < tail_start) ? a.log2B : a.log2T, a.c_hi, a.c_lo) : 0.f;
+      }
+      switch (c0 / kChunk) {
+#define RQ_KEEP(n)                                                            \
+  case n:                                                                     \
+    kept[n][0] = v[0]; kept[n][1] = v[1]; kept[n][2] = v[2]; kept[n][3] = v[3]; \
+    kept_L[n] = L;                                                            \
+    break;
+        RQ_KEEP(0)
+        RQ_KEEP(1)
+        default:
+          kept[2][0] = v[0]; kept[2][1] = v[1]; kept[2][2] = v[2]; kept[2][3] = v[3];
+          kept_L[2] = L;
+          break;
+#undef RQ_KEEP
+      }
+    }
+    if (len == kChunk && c0 + len <= tail_start) {   // every value is in a block of size B
+#pragma unroll
+      for (int e = 0; e < 16; ++e) {
+        const long long v = f[e] < 0 ? -f[e] : f[e];
+        mB = v > mB ? v : mB;
+      }
+    } else {
+#pragma unroll
+      for (int e = 0; e < 16; ++e) {
+        const int i = rq_pos(L, tid, e);
+        if (i < len) {
+          const long long v = f[e] < 0 ? -f[e] : f[e];
+          if (c0 + i < tail_start)
+            mB = v > mB ? v : mB;
+          else
+            mT = v > mT ? v : mT;
+        }
+      }
+    }
+  }
+  if (tid == 0) DPTQ_TRACE_CLOCK(tr, 140);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const long long b = __shfl_xor_sync(0xffffffffu, mB, o), t = __shfl_xor_sync(0xffffffffu, mT, o);
+    mB = b > mB ? b : mB;
+    mT = t > mT ? t : mT;
+  }
+  if ((tid & 31) == 0) {
+    red[tid >> 5] = mB;
+    red[8 + (tid >> 5)] = mT;
+  }
+  sync();
+#pragma unroll
+  for (int w = 0; w < kRQThreads / 32; ++w) {
+    mB = red[w] > mB ? red[w] : mB;
+    mT = red[8 + w] > mT ? red[8 + w] : mT;
+  }
+  const float yB = mB ? fixed_to_rotated(mB, a.log2B, a.c_hi, a.c_lo) : 0.f;
+  const float yT = mT ? fixed_to_rotated(mT, a.log2T, a.c_hi, a.c_lo) : 0.f;
+  const float amax = fmaxf(yB, yT);
+  const float s = __fdiv_rn(amax, qmaxf);
+  const bool nz = amax > 0.f;
+  const float rs = nz ? __frcp_rn(s) : 0.f;
+  if (part == 0 && tid == 0 && a.scales != nullptr) a.scales[row] = nz ? s : 0.f;
+  if (tid == 0) DPTQ_TRACE_CLOCK(tr, 141);
+
+  // ---- pass 2: this part's codes, chunk by chunk
+  const int elo = 16 * part / np, ehi = 16 * (part + 1) / np;
+  for (int c0 = 0; c0 < K; c0 += kChunk) {
+    const int len = min(kChunk, K - c0);
+    const int ch = c0 / kChunk;
+    int L = L0;
+    if (keep)
+      L = ch == 0 ? kept_L[0] : ch == 1 ? kept_L[1] : kept_L[2];
+    else if (K > kChunk)
+      L = rq_chunk(a, src, c0, len, tail_start, f, sx, tid, sync);
+#pragma unroll 1
+    for (int g4 = elo >> 2; g4 < ehi >> 2; ++g4) {   // this part's values, 4 at a time
+      int idx[4];
+      float y[4], c[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int j = 0; j < 4; ++j) idx[j] = rq_pos(L, tid, 4 * g4 + j);
+      if (keep) {
+        switch (ch) {
+          case 0: y[0] = kept[0][0]; y[1] = kept[0][1]; y[2] = kept[0][2]; y[3] = kept[0][3]; break;
+          case 1: y[0] = kept[1][0]; y[1] = kept[1][1]; y[2] = kept[1][2]; y[3] = kept[1][3]; break;
+          default: y[0] = kept[2][0]; y[1] = kept[2][1]; y[2] = kept[2][2]; y[3] = kept[2][3]; break;
+        }
+      } else {
+        long long v[4];
+        switch (g4) {
+          case 0: v[0] = f[0]; v[1] = f[1]; v[2] = f[2]; v[3] = f[3]; break;
+          case 1: v[0] = f[4]; v[1] = f[5]; v[2] = f[6]; v[3] = f[7]; break;
+          case 2: v[0] = f[8]; v[1] = f[9]; v[2] = f[10]; v[3] = f[11]; break;
+          default: v[0] = f[12]; v[1] = f[13]; v[2] = f[14]; v[3] = f[15]; break;
+        }
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          y[j] = idx[j] < len ? fixed_to_rotated(v[j], (c0 + idx[j] < tail_start) ? a.log2B : a.log2T, a.c_hi, a.c_lo)
+                              : 0.f;
+      }
+      if (nz) quant_code4(y, s, rs, qminf, qmaxf, c);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        if (idx[j] < len) {
+          if (bits == 4) {
+            cst[idx[j]] = (uint8_t)e4m3_byte(c[j]);
+          } else {
+            const float m = fabsf(c[j]);
+            const float h = __fmul_rn(floorf(__fmul_rn(m, 0.0625f)), 16.f);
+            cst[idx[j]] = (uint8_t)e4m3_byte(__fadd_rn(copysignf(h, c[j]), 0.0f));
+            cst[kChunk + idx[j]] = (uint8_t)e4m3_byte(__fadd_rn(copysignf(__fsub_rn(m, h), c[j]), 0.0f));
+          }
+        }
+      }
+    }
+    if (tid == 0 && c0 == 0) DPTQ_TRACE_CLOCK(tr, 142);
+    sync();
+    for (int w = tid; w < len / 4; w += kRQThreads) {
+      const int i = 4 * w;
+      const int ei = L == 2 ? i >> 8 : L == 1 ? (i >> 4) & 15 : i & 15;
+      if (ei >= elo && ei < ehi)
+        store4(c0 + i, *reinterpret_cast<const uint32_t*>(cst + i),
+               *reinterpret_cast<const uint32_t*>(cst + kChunk + i));
+    }
+    if (tid == 0 && c0 == 0) DPTQ_TRACE_CLOCK(tr, 143);
+    sync();   // the staging buffer is reused by the next chunk
+  }
+  if (part == np - 1)   // k in [K, K_pad): zero codes
+    for (int k = K + 4 * tid; k < K_pad; k += 4 * kRQThreads) store4(k, 0u, 0u);
 }
 
 }  // namespace dptq
