@@ -73,6 +73,18 @@ def _load():
             lib.orc_unpack_nibbles.restype = None
             lib.orc_residual_stats.argtypes = [P, P, I, I, I, ctypes.c_double, P, P]
             lib.orc_residual_stats.restype = I
+            lib.orc_rotate_f16_signed.argtypes = [P, P, I, I, I, P]
+            lib.orc_rotate_f16_signed.restype = I
+            lib.orc_rotate_quant_act_signed.argtypes = [P, I, I, I, I, P, P, P]
+            lib.orc_rotate_quant_act_signed.restype = I
+            lib.orc_pack_weights_signed.argtypes = [P, I, I, I, P, P, P]
+            lib.orc_pack_weights_signed.restype = I
+            lib.orc_qlinear_signed.argtypes = [P, I, I, I, I, P, P, P, I, P, P, P, P]
+            lib.orc_qlinear_signed.restype = I
+            lib.orc_kv4_quantize.argtypes = [P, I, I, I, P, P]
+            lib.orc_kv4_quantize.restype = I
+            lib.orc_policy_mask.argtypes = [P, P, I, ctypes.c_double, ctypes.c_double, P]
+            lib.orc_policy_mask.restype = None
             _lib = lib
     return _lib
 
@@ -118,12 +130,22 @@ def rotate_row_f64(x: np.ndarray, B: int) -> np.ndarray:
     return y
 
 
-def rotate(x_f16: np.ndarray, B: int) -> np.ndarray:
-    """fp16 [M, K] -> fp32 [M, K]: x R with R = blockdiag(H/sqrt(block)) (Eq. 4)."""
+def _signs(signs, K):
+    if signs is None:
+        return None
+    d = np.ascontiguousarray(signs, dtype=np.int8)
+    assert d.shape == (K,) and np.all(np.abs(d) == 1), "signs must be K values of +1 / -1"
+    return d
+
+
+def rotate(x_f16: np.ndarray, B: int, signs=None) -> np.ndarray:
+    """fp16 [M, K] -> fp32 [M, K]: x R with R = blockdiag(H/sqrt(block)) (Eq. 4); with
+    `signs` (K values of +-1) the randomized Hadamard x diag(signs) R."""
     xb = _as_half_bits(x_f16)
     M, K = xb.shape
     y = np.empty((M, K), dtype=np.float32)
-    if not _load().orc_rotate_f16(_p(xb), _p(y), M, K, B):
+    d = _signs(signs, K)
+    if not _load().orc_rotate_f16_signed(_p(xb), _p(y), M, K, B, None if d is None else _p(d)):
         raise ValueError("bad block layout")
     return y
 
@@ -139,23 +161,25 @@ def quant_rows(y: np.ndarray, bits: int):
     return c, s
 
 
-def rotate_quant_act(x_f16: np.ndarray, B: int, bits: int):
+def rotate_quant_act(x_f16: np.ndarray, B: int, bits: int, signs=None):
     xb = _as_half_bits(x_f16)
     M, K = xb.shape
     c = np.empty((M, K), dtype=np.int8)
     s = np.empty((M,), dtype=np.float32)
-    if not _load().orc_rotate_quant_act(_p(xb), M, K, B, bits, _p(c), _p(s)):
+    d = _signs(signs, K)
+    if not _load().orc_rotate_quant_act_signed(_p(xb), M, K, B, bits, None if d is None else _p(d), _p(c), _p(s)):
         raise ValueError("bad shape or bits")
     return c, s
 
 
-def pack_weights(W_f16: np.ndarray, B: int):
+def pack_weights(W_f16: np.ndarray, B: int, signs=None):
     """RTN int4 per-channel symmetric weights with R folded in (Eq. 5): (q int8 [N,K], s_w fp32 [N])."""
     wb = _as_half_bits(W_f16)
     N, K = wb.shape
     q = np.empty((N, K), dtype=np.int8)
     s = np.empty((N,), dtype=np.float32)
-    if not _load().orc_pack_weights(_p(wb), N, K, B, _p(q), _p(s)):
+    d = _signs(signs, K)
+    if not _load().orc_pack_weights_signed(_p(wb), N, K, B, None if d is None else _p(d), _p(q), _p(s)):
         raise ValueError("bad shape")
     return q, s
 
@@ -182,7 +206,7 @@ def epilogue(acc: np.ndarray, sa: np.ndarray, sw: np.ndarray) -> np.ndarray:
     return out.view(np.float16)
 
 
-def qlinear(x_f16: np.ndarray, B: int, bits: int, q: np.ndarray, sw: np.ndarray):
+def qlinear(x_f16: np.ndarray, B: int, bits: int, q: np.ndarray, sw: np.ndarray, signs=None):
     """Whole layer: returns dict(out fp16 [M,N], acc int32, codes int8, sa fp32)."""
     xb = _as_half_bits(x_f16)
     M, K = xb.shape
@@ -193,8 +217,9 @@ def qlinear(x_f16: np.ndarray, B: int, bits: int, q: np.ndarray, sw: np.ndarray)
     acc = np.empty((M, N), dtype=np.int32)
     codes = np.empty((M, K), dtype=np.int8)
     sa = np.empty((M,), dtype=np.float32)
-    if not _load().orc_qlinear(_p(xb), M, K, B, bits, _p(q), _p(sw), N, _p(out), _p(acc),
-                               _p(codes), _p(sa)):
+    d = _signs(signs, K)
+    if not _load().orc_qlinear_signed(_p(xb), M, K, B, bits, None if d is None else _p(d), _p(q), _p(sw), N,
+                                      _p(out), _p(acc), _p(codes), _p(sa)):
         raise ValueError("bad shape, bits or int32 overflow")
     return {"out": out.view(np.float16), "acc": acc, "codes": codes, "sa": sa}
 
@@ -227,3 +252,26 @@ def residual_stats(x: np.ndarray, dx: np.ndarray, bits: int, eps: float = 1e-6):
                                       ctypes.byref(snr)):
         raise MemoryError
     return jr.value, snr.value
+
+
+def kv4_quantize(x_f16: np.ndarray, group: int = 128):
+    """Group-wise symmetric 4-bit KV-cache codes (Section 4.2, group 128):
+    (codes int8 [rows, cols], scales fp32 [rows, cols // group])."""
+    xb = _as_half_bits(x_f16)
+    R, C = xb.shape
+    c = np.empty((R, C), dtype=np.int8)
+    s = np.empty((R, C // group if group > 0 else 0), dtype=np.float32)
+    if not _load().orc_kv4_quantize(_p(xb), R, C, group, _p(c), _p(s)):
+        raise ValueError("group must divide the number of columns")
+    return c, s
+
+
+def policy_mask(jr, snr, tau_jr: float, tau_snr: float) -> np.ndarray:
+    """Per-layer activation bits (Section 3.3 Eq. 20, Algorithm 1 step 2): 8 on the
+    sensitive set {l: JR_l > tau_jr and SNR_l < tau_snr}, else 4."""
+    jr = np.ascontiguousarray(jr, dtype=np.float64)
+    snr = np.ascontiguousarray(snr, dtype=np.float64)
+    L = jr.shape[0]
+    bits = np.empty((L,), dtype=np.uint8)
+    _load().orc_policy_mask(_p(jr), _p(snr), L, tau_jr, tau_snr, _p(bits))
+    return bits

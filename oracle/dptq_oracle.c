@@ -140,21 +140,32 @@ int orc_rotate_row_f64(const double* x, double* y, int K, int B) {
 }
 
 /* Rotate an fp16 matrix x[M][K] (row-major, raw binary16 bits) into fp32 y[M][K]:
- * evaluate in fp64, round once to fp32. */
-int orc_rotate_f16(const uint16_t* x, float* y, int M, int K, int B) {
+ * evaluate in fp64, round once to fp32.
+ * signs (may be NULL): the randomized Hadamard of QuaRot (Section 1; Section 4.2),
+ * R' = D R with D = diag(signs), signs[k] in {+1, -1}: x is multiplied elementwise by
+ * the signs before the block Hadamard.  D is orthogonal, so R'^T R' = I still holds
+ * (Eq. 4), and folding the same R' into the weights keeps X W^T (Eq. 5). */
+int orc_rotate_f16_signed(const uint16_t* x, float* y, int M, int K, int B, const int8_t* signs) {
     int q, r;
     if (!orc_block_layout(K, B, &q, &r)) return 0;
     double* xr = (double*)malloc(sizeof(double) * (size_t)K);
     double* yr = (double*)malloc(sizeof(double) * (size_t)K);
     if (!xr || !yr) { free(xr); free(yr); return 0; }
     for (int m = 0; m < M; ++m) {
-        for (int k = 0; k < K; ++k) xr[k] = orc_half_to_double(x[(size_t)m * K + k]);
+        for (int k = 0; k < K; ++k) {
+            xr[k] = orc_half_to_double(x[(size_t)m * K + k]);
+            if (signs && signs[k] < 0) xr[k] = -xr[k];
+        }
         orc_rotate_row_f64(xr, yr, K, B);
         for (int k = 0; k < K; ++k) y[(size_t)m * K + k] = (float)yr[k];
     }
     free(xr);
     free(yr);
     return 1;
+}
+
+int orc_rotate_f16(const uint16_t* x, float* y, int M, int K, int B) {
+    return orc_rotate_f16_signed(x, y, M, K, B, NULL);
 }
 
 /* ------------------------------------------------------------------------- */
@@ -193,22 +204,32 @@ int orc_quant_rows(const float* y, int M, int K, int bits, int8_t* codes, float*
     return 1;
 }
 
-/* Online activation path: rotate (Eq. 4) then per-token quantize (Eq. 2). */
-int orc_rotate_quant_act(const uint16_t* x, int M, int K, int B, int bits,
-                         int8_t* codes, float* scales) {
+/* Online activation path: rotate (Eq. 4) then per-token quantize (Eq. 2).
+ * signs: NULL, or the randomized Hadamard's diagonal (see orc_rotate_f16_signed). */
+int orc_rotate_quant_act_signed(const uint16_t* x, int M, int K, int B, int bits, const int8_t* signs,
+                                int8_t* codes, float* scales) {
     if (bits != 4 && bits != 8) return 0;
     float* y = (float*)malloc(sizeof(float) * (size_t)M * K);
     if (!y) return 0;
-    int ok = orc_rotate_f16(x, y, M, K, B);
+    int ok = orc_rotate_f16_signed(x, y, M, K, B, signs);
     if (ok) orc_quant_rows(y, M, K, bits, codes, scales);
     free(y);
     return ok;
 }
 
+int orc_rotate_quant_act(const uint16_t* x, int M, int K, int B, int bits,
+                         int8_t* codes, float* scales) {
+    return orc_rotate_quant_act_signed(x, M, K, B, bits, NULL, codes, scales);
+}
+
 /* Offline weight path (Eq. 5 fold, Section 4.2 RTN per-channel symmetric int4):
  * W'[n] = W[n] R, s_w[n] = max|W'[n]| / 7, q = clamp(rint(W'/s_w), -8, 7). */
+int orc_pack_weights_signed(const uint16_t* W, int N, int K, int B, const int8_t* signs, int8_t* q, float* sw) {
+    return orc_rotate_quant_act_signed(W, N, K, B, 4, signs, q, sw);
+}
+
 int orc_pack_weights(const uint16_t* W, int N, int K, int B, int8_t* q, float* sw) {
-    return orc_rotate_quant_act(W, N, K, B, 4, q, sw);
+    return orc_pack_weights_signed(W, N, K, B, NULL, q, sw);
 }
 
 /* ------------------------------------------------------------------------- */
@@ -248,20 +269,64 @@ void orc_epilogue(const int32_t* acc, const float* sa, const float* sw, int M, i
 /* The whole quantized linear layer for one activation matrix:
  * rotate + quantize x, integer GEMM against packed weights q (int4 codes in int8),
  * scale epilogue.  acc may be NULL.  Returns 0 on a bad shape or int32 overflow. */
-int orc_qlinear(const uint16_t* x, int M, int K, int B, int bits,
-                const int8_t* q, const float* sw, int N,
-                uint16_t* out, int32_t* acc_out, int8_t* codes_out, float* sa_out) {
+int orc_qlinear_signed(const uint16_t* x, int M, int K, int B, int bits, const int8_t* signs,
+                       const int8_t* q, const float* sw, int N,
+                       uint16_t* out, int32_t* acc_out, int8_t* codes_out, float* sa_out) {
     int8_t* codes = codes_out ? codes_out : (int8_t*)malloc((size_t)M * K);
     float* sa = sa_out ? sa_out : (float*)malloc(sizeof(float) * (size_t)M);
     int32_t* acc = acc_out ? acc_out : (int32_t*)malloc(sizeof(int32_t) * (size_t)M * N);
     int ok = codes && sa && acc;
-    if (ok) ok = orc_rotate_quant_act(x, M, K, B, bits, codes, sa);
+    if (ok) ok = orc_rotate_quant_act_signed(x, M, K, B, bits, signs, codes, sa);
     if (ok) ok = orc_gemm_i32(codes, q, M, N, K, acc);
     if (ok) orc_epilogue(acc, sa, sw, M, N, out);
     if (!codes_out) free(codes);
     if (!sa_out) free(sa);
     if (!acc_out) free(acc);
     return ok;
+}
+
+int orc_qlinear(const uint16_t* x, int M, int K, int B, int bits,
+                const int8_t* q, const float* sw, int N,
+                uint16_t* out, int32_t* acc_out, int8_t* codes_out, float* sa_out) {
+    return orc_qlinear_signed(x, M, K, B, bits, NULL, q, sw, N, out, acc_out, codes_out, sa_out);
+}
+
+/* ------------------------------------------------------------------------- */
+/* KV-cache quantization (Section 4.2: group-wise, group size 128, 4-bit)       */
+/* ------------------------------------------------------------------------- */
+
+/* Group-wise symmetric 4-bit codes of an fp16 matrix x[rows][cols]: each row is cut
+ * into groups of `group` consecutive columns, and each group is quantized on its own
+ * with the quantizer of Eq. 2 (s = max|x| / 7, c = clamp(rint(x / s), -8, 7), an
+ * all-zero group gets s = 0).  The paper says group-wise with group 128 and does not
+ * say symmetric or asymmetric; symmetric is this oracle's reading.  codes int8
+ * [rows][cols], scales fp32 [rows][cols / group].  Returns 0 unless group divides
+ * cols. */
+int orc_kv4_quantize(const uint16_t* x, int rows, int cols, int group, int8_t* codes, float* scales) {
+    if (group <= 0 || cols % group != 0) return 0;
+    float* v = (float*)malloc(sizeof(float) * (size_t)group);
+    if (!v) return 0;
+    int ng = cols / group;
+    for (int m = 0; m < rows; ++m) {
+        for (int g = 0; g < ng; ++g) {
+            size_t base = (size_t)m * cols + (size_t)g * group;
+            for (int i = 0; i < group; ++i) v[i] = (float)orc_half_to_double(x[base + i]);
+            scales[(size_t)m * ng + g] = orc_quant_row(v, group, 4, codes + base);
+        }
+    }
+    free(v);
+    return 1;
+}
+
+/* ------------------------------------------------------------------------- */
+/* Sensitive-layer policy (Section 3.3, Eq. 20; Algorithm 1 step 2)             */
+/* ------------------------------------------------------------------------- */
+
+/* bits[l] = 8 if JR_l > tau_jr and SNR_l < tau_snr (the sensitive set of Eq. 20),
+ * else 4.  The paper gives no threshold values; they are inputs. */
+void orc_policy_mask(const double* jr, const double* snr, int L, double tau_jr, double tau_snr,
+                     uint8_t* bits) {
+    for (int l = 0; l < L; ++l) bits[l] = (jr[l] > tau_jr && snr[l] < tau_snr) ? 8 : 4;
 }
 
 /* ------------------------------------------------------------------------- */

@@ -338,3 +338,110 @@ def test_sensitive_set_golden():
             (ln.split("|") for ln in _rows("sensitive_set.txt"))}
     for L, layers in gold.items():
         assert layers == [0, 1, 2, L - 1]
+
+
+# ---------------------------------------------------------------- randomized Hadamard
+def _signs(K, seed):
+    return np.where(np.random.default_rng(seed).random(K) < 0.5, -1, 1).astype(np.int8)
+
+
+def test_randomized_hadamard_all_plus_signs_is_plain(orc):
+    x = inputs.to_f16(np.random.default_rng(40).standard_normal((5, 768)).astype(np.float32))
+    assert np.array_equal(orc.rotate(x, 256, signs=np.ones(768, np.int8)), orc.rotate(x, 256))
+    c0, s0 = orc.rotate_quant_act(x, 256, 4)
+    c1, s1 = orc.rotate_quant_act(x, 256, 4, signs=np.ones(768, np.int8))
+    assert np.array_equal(c0, c1) and np.array_equal(s0, s1)
+
+
+def test_randomized_hadamard_brute_force(orc):
+    # y = (x * d) blockdiag(H_8, H_8, H_4) / sqrt(block) with the textbook Sylvester matrix:
+    # the fp16 inputs make every fp64 sum exact, so the fp32 results agree bit for bit.
+    K, B = 20, 8
+    x = inputs.to_f16(np.random.default_rng(41).standard_normal((3, K)).astype(np.float32))
+    d = _signs(K, 42)
+    xs = x.astype(np.float64) * d
+    R = np.zeros((K, K))
+    R[0:8, 0:8] = sylvester(8) / math.sqrt(8)
+    R[8:16, 8:16] = sylvester(8) / math.sqrt(8)
+    R[16:20, 16:20] = sylvester(4) / math.sqrt(4)
+    ref = (xs @ R).astype(np.float32)
+    assert np.array_equal(orc.rotate(x, B, signs=d), ref)
+    # a sign flip is a sign flip of the input element (and nothing else)
+    d2 = d.copy()
+    d2[5] = -d2[5]
+    x2 = x.copy()
+    x2[:, 5] = -x2[:, 5]
+    assert np.array_equal(orc.rotate(x2, B, signs=d2), orc.rotate(x, B, signs=d))
+
+
+def test_randomized_hadamard_is_orthogonal_and_folds_into_weights(orc):
+    K, B = 512, 128
+    rng = np.random.default_rng(43)
+    d = _signs(K, 44)
+    x = inputs.to_f16(rng.standard_normal((4, K)).astype(np.float32))
+    W = inputs.to_f16((0.02 * rng.standard_normal((6, K))).astype(np.float32))
+    y = orc.rotate(x, B, signs=d).astype(np.float64)
+    yw = orc.rotate(W, B, signs=d).astype(np.float64)
+    xf, wf = x.astype(np.float64), W.astype(np.float64)
+    assert np.allclose(np.linalg.norm(y, axis=1), np.linalg.norm(xf, axis=1), rtol=1e-6)   # (DR)^T DR = I
+    assert np.allclose(y @ yw.T, xf @ wf.T, rtol=1e-5, atol=1e-6)                          # Eq. 5 with R' = DR
+    # a different sign vector gives a different rotation
+    assert not np.array_equal(orc.rotate(x, B, signs=_signs(K, 45)), orc.rotate(x, B, signs=d))
+
+
+def test_randomized_hadamard_weights_and_layer(orc):
+    K, B, N, M = 256, 64, 32, 5
+    rng = np.random.default_rng(46)
+    d = _signs(K, 47)
+    W = inputs.to_f16((0.02 * rng.standard_normal((N, K))).astype(np.float32))
+    x = inputs.to_f16(rng.standard_normal((M, K)).astype(np.float32))
+    q, sw = orc.pack_weights(W, B, signs=d)
+    qc, sc = orc.rotate_quant_act(W, B, 4, signs=d)
+    assert np.array_equal(q, qc) and np.array_equal(sw, sc)
+    r = orc.qlinear(x, B, 8, q, sw, signs=d)
+    codes, sa = orc.rotate_quant_act(x, B, 8, signs=d)
+    assert np.array_equal(r["codes"], codes) and np.array_equal(r["sa"], sa)
+    assert np.array_equal(r["acc"], codes.astype(np.int64) @ q.astype(np.int64).T)
+    assert np.array_equal(r["out"].view(np.uint16), orc.epilogue(r["acc"], sa, sw).view(np.uint16))
+
+
+# ---------------------------------------------------------------- KV4 quantizer
+def test_kv4_golden_worked_examples(orc):
+    for ln in _rows("kv4_worked.txt"):
+        g, xs, s, cs = [p.strip() for p in ln.split("|")]
+        x = inputs.to_f16(np.array([[float(v) for v in xs.split()]], dtype=np.float32))
+        codes, scales = orc.kv4_quantize(x, int(g))
+        assert scales[0, 0] == np.float32(float(s))
+        assert codes[0].tolist() == [int(v) for v in cs.split()]
+
+
+def test_kv4_groups_are_independent_and_bounded(orc):
+    rng = np.random.default_rng(48)
+    x = inputs.to_f16((rng.standard_normal((6, 512)) * np.float32(3.0) ** rng.integers(-3, 4, (6, 1))).astype(np.float32))
+    x[2, 128:256] = 0                                          # an all-zero group
+    codes, scales = orc.kv4_quantize(x, 128)
+    assert codes.shape == (6, 512) and scales.shape == (6, 4)
+    xf = x.astype(np.float32).reshape(6, 4, 128)
+    c = codes.reshape(6, 4, 128).astype(np.float32)
+    assert np.all(np.abs(codes) <= 7)                          # symmetric: -8 is never produced
+    assert np.all(scales == np.max(np.abs(xf), axis=2) / np.float32(7))
+    err = np.abs(xf - scales[:, :, None] * c)
+    assert np.all(err <= scales[:, :, None] * 0.5 * (1 + 1e-6))   # round-trip error <= s/2
+    assert scales[2, 1] == 0 and np.all(codes[2, 128:256] == 0)
+    # each group is the per-token quantizer of Eq. 2 applied to that group alone
+    for gi in range(4):
+        cg, sg = orc.quant_rows(xf[:, gi, :], 4)
+        assert np.array_equal(cg, codes[:, gi * 128:(gi + 1) * 128]) and np.array_equal(sg, scales[:, gi])
+    with pytest.raises(ValueError):
+        orc.kv4_quantize(x[:, :200], 128)
+
+
+# ---------------------------------------------------------------- sensitive-layer policy
+def test_policy_mask_closed_form(orc):
+    jr = np.array([0.9, 0.9, 0.1, 0.5, 0.5, 0.3], dtype=np.float64)
+    snr = np.array([5.0, 25.0, 5.0, 20.0, 19.0, 10.0], dtype=np.float64)
+    bits = orc.policy_mask(jr, snr, tau_jr=0.3, tau_snr=20.0)
+    # Eq. 20: JR > tau_JR and SNR < tau_SNR, both strict (layer 3 has SNR == tau, layer 5 JR == tau)
+    assert bits.tolist() == [8, 4, 4, 4, 8, 4]
+    assert orc.policy_mask(jr, snr, tau_jr=-1.0, tau_snr=1e9).tolist() == [8] * 6
+    assert orc.policy_mask(jr, snr, tau_jr=1.0, tau_snr=1e9).tolist() == [4] * 6
