@@ -439,9 +439,36 @@ def run_shapes(args):
             h.close()
         del hs
         torch.cuda.synchronize()
+    # KV4 group-128 quantizer over one layer's K cache (LLaMA-2-7B, 32 heads x 128, 8192
+    # tokens: 64 MB fp16) and the sensitivity policy over 32 layers x 512 tokens x 4096
+    # (2 x 268 MB fp32): both HBM-bound; inputs rotated through copies beyond 2x L2.
+    extra = []
+    T, H, D = 8192, 32, 128
+    kvs = [torch.from_numpy(inputs.activations(inputs.llama2_7b_decode(), 1024, 128)).to(dev).repeat(T * H // 1024, 1)
+           for _ in range(3)]
+    codes = torch.empty((T * H, D // 2), dtype=torch.uint8, device=dev)
+    sc = torch.empty((T * H, 1), dtype=torch.float32, device=dev)
+    t_kv = t_graph([lambda kv=kv: dptq.dptq_kv4_quantize(kv, 128, codes, sc, stream=stream) for kv in kvs])
+    kv_b = T * H * D * 2 + T * H * D // 2 + T * H * 4
+    extra.append({"kernel": "kv4_quantize", "rows": T * H, "cols": D, "group": 128, "us": t_kv,
+                  "gbs": kv_b / t_kv / 1e3, "roofline": {"bound": "hbm", "peak_gbs": hbm, "frac": kv_b / t_kv / 1e3 / hbm}})
+    del kvs, codes, sc
+    L, TT, d = 32, 512, 4096
+    g = torch.Generator(device=dev).manual_seed(9)
+    xs = torch.randn((L, TT, d), generator=g, device=dev)
+    dxs = 0.1 * torch.randn((L, TT, d), generator=g, device=dev)
+    jr = torch.empty((L,), dtype=torch.float64, device=dev)
+    snr = torch.empty((L,), dtype=torch.float64, device=dev)
+    bo = torch.empty((L,), dtype=torch.uint8, device=dev)
+    t_pol = t_graph([lambda: dptq.dptq_sensitivity_policy(xs, dxs, 4, 1e-6, 0.1, 20.0, jr, snr, bo, stream=stream)])
+    pol_b = 2 * L * TT * d * 4
+    extra.append({"kernel": "sensitivity_policy", "L": L, "T": TT, "d": d, "us": t_pol, "gbs": pol_b / t_pol / 1e3,
+                  "roofline": {"bound": "hbm", "peak_gbs": hbm, "frac": pol_b / t_pol / 1e3 / hbm}})
+    print(f"[shapes] kv4 {t_kv:.1f} us, policy {t_pol:.1f} us", file=sys.stderr, flush=True)
     dptq.dptq_last_device_error()
     print(json.dumps({"mode": "shapes", "timing": "CUDA events over graph replays, weights rotated through "
-                                                  ">= 2x L2 of copies", "shapes": rows}), flush=True)
+                                                  ">= 2x L2 of copies", "shapes": rows, "extra_kernels": extra}),
+          flush=True)
     return 0
 
 

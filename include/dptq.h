@@ -79,6 +79,15 @@ typedef struct dptq_linear* dptq_handle;
 dptq_status dptq_pack_weights(const void* W_fp16, int N, int K, int had_block, int w_on_device,
                               dptq_handle* out);
 
+/* Randomized Hadamard variant (QuaRot's rotation, named in Section 1 and Section 4.2):
+ * R' = D R with D = diag(signs), signs_host[k] in {+1, -1} for k < K (host memory, read
+ * only, copied into the handle).  D is orthogonal, so R'^T R' = I (Eq. 4) and folding
+ * R' into W keeps X W^T (Eq. 5).  Packs W' = W R' like dptq_pack_weights; every
+ * qlinear call on the returned handle then rotates x by the same R'.  INVALID_ARG if a
+ * sign is neither +1 nor -1. */
+dptq_status dptq_pack_weights_rh(const void* W_fp16, int N, int K, int had_block, const int8_t* signs_host,
+                                 int w_on_device, dptq_handle* out);
+
 /* Online rotation + quantization of activations (Section 2 Eq. 4 then Eq. 2).
  * x_fp16: device [M][K] binary16.  bits: 4 or 8 (the mask entry of the layer).
  * codes (device, written): bits == 4: uint8 [M][K/2], byte j of a row holds code 2j in
@@ -94,6 +103,45 @@ dptq_status dptq_rotate_quant_act(const void* x_fp16, int M, int K, int had_bloc
  * quantizer of dptq_rotate_quant_act sees. */
 dptq_status dptq_rotate_act(const void* x_fp16, int M, int K, int had_block, float* y_f32,
                             void* stream);
+
+/* dptq_rotate_quant_act and dptq_rotate_act with the randomized Hadamard R' = D R:
+ * signs_dev is a DEVICE array of K int8 values, 16-byte aligned (a value below zero
+ * means -1, any other +1), or NULL for the plain block Hadamard.  INVALID_ARG if
+ * signs_dev is not 16-byte aligned. */
+dptq_status dptq_rotate_quant_act_rh(const void* x_fp16, int M, int K, int had_block, int bits,
+                                     const int8_t* signs_dev, void* codes, float* scales, void* stream);
+dptq_status dptq_rotate_act_rh(const void* x_fp16, int M, int K, int had_block, const int8_t* signs_dev,
+                               float* y_f32, void* stream);
+
+/* KV-cache quantization (Section 4.2: "group-wise quantization with a group size of
+ * 128", 4 bits).  kv_fp16: device [rows][cols] binary16 (16-byte aligned).  Each row is
+ * cut into groups of `group` consecutive columns, each quantized on its own,
+ * symmetrically (the paper does not say symmetric or asymmetric): s = max|x| / 7 in
+ * fp32 (IEEE division), c = clamp(round-half-even(x / s), -8, 7) (never -8), an
+ * all-zero group has s = 0 and codes 0.
+ * codes (device, written): uint8 [rows][cols/2] in the A4 format of
+ * dptq_rotate_quant_act (low nibble = even column); scales (device, written): float
+ * [rows][cols / group].  group: a multiple of 128 up to 1024 that divides cols (the
+ * paper's 128).  Asynchronous.  INVALID_ARG for null pointers, negative sizes or a
+ * misaligned kv_fp16; UNSUPPORTED for other group sizes.  rows == 0 is a no-op. */
+dptq_status dptq_kv4_quantize(const void* kv_fp16, int rows, int cols, int group, void* codes, float* scales,
+                              void* stream);
+
+/* Sensitive-layer policy: the statistics of Section 3.1 and the set of Section 3.3
+ * (Eq. 20), giving the activation bits of Algorithm 1 step 2.  For layer l with
+ * residual state x_t (entering the layer) and update dx_t of token t:
+ *   Jump Ratio        JR_l  = mean_t ||dx_t|| / (||x_t|| + eps)                 (Eqs. 8-9)
+ *   historical SNR    SNR_l = mean_t 10 log10(||x_t||^2 / (||xhat_t - x_t||^2 + eps)),
+ *                     xhat_t = Q_b(x_t + dx_t) - dx_t, Q_b the per-token symmetric
+ *                     quantizer at `bits` on the fp32 sum x_t + dx_t     (Eqs. 10-11)
+ *   bits_out[l] = 8 if JR_l > tau_jr and SNR_l < tau_snr, else 4.          (Eq. 20)
+ * x, dx: device fp32 [L][T][d], 16-byte aligned, d % 4 == 0; jr, snr: device double
+ * [L] (written); bits_out: device uint8 [L] (written).  bits in {4, 8}; eps >= 0 (the
+ * paper's epsilon; its value is not given).  Norms and errors are evaluated in fp32 per
+ * element and summed in fp64 per token.  Asynchronous. */
+dptq_status dptq_sensitivity_policy(const float* x, const float* dx, int L, int T, int d, int bits, double eps,
+                                    double tau_jr, double tau_snr, double* jr, double* snr, uint8_t* bits_out,
+                                    void* stream);
 
 /* The quantized linear layer: out = fp16( Q(x R) (W R)^T scaled ), i.e. rotate and
  * quantize x with `bits` (4 or 8, the layer's mask entry), multiply by the packed

@@ -22,7 +22,7 @@ TRACE = os.environ.get("DPTQ_TRACE") == "1"
 if TRACE:
     OUT_DIR = os.path.join(HERE, "_build_trace")
     LIB = os.path.join(OUT_DIR, "libdptq.so")
-SOURCES = ["api.cu", "rotate_quant.cu", "qgemm.cu", "static_scratch.cu"]
+SOURCES = ["api.cu", "rotate_quant.cu", "qgemm.cu", "static_scratch.cu", "kv_policy.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

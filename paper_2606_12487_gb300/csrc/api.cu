@@ -229,7 +229,10 @@ const char* dptq_status_str(dptq_status s) {
 
 const char* dptq_last_error_message(void) { return g_msg.c_str(); }
 
-dptq_status dptq_pack_weights(const void* W_fp16, int N, int K, int had_block, int w_on_device, dptq_handle* out) {
+namespace {
+// Shared body of dptq_pack_weights and dptq_pack_weights_rh (signs_host null: plain).
+dptq_status pack_weights_impl(const void* W_fp16, int N, int K, int had_block, const int8_t* signs_host,
+                              int w_on_device, dptq_handle* out) {
   if (!W_fp16 || !out) return fail(DPTQ_ERR_INVALID_ARG, "null pointer");
   *out = nullptr;
   if (N <= 0 || K <= 0 || had_block <= 0) return fail(DPTQ_ERR_INVALID_ARG, "sizes must be positive");
@@ -248,10 +251,22 @@ dptq_status dptq_pack_weights(const void* W_fp16, int N, int K, int had_block, i
   h->KB = h->K_pad / kKBlock;
   h->N_pad = round_up(N, 128);
   h->had_block = had_block;
+  if (signs_host != nullptr) {
+    for (int k = 0; k < K; ++k)
+      if (signs_host[k] != 1 && signs_host[k] != -1) {
+        delete h;
+        return fail(DPTQ_ERR_INVALID_ARG, "signs must be +1 or -1");
+      }
+  }
   const size_t wt_bytes = (size_t)(h->N_pad / 128) * h->KB * kWTileBytes;
   void* tmp = nullptr;
   cudaError_t e = cudaMalloc(&h->wt, wt_bytes);
   if (e == cudaSuccess) e = cudaMalloc(&h->sw, sizeof(float) * h->N_pad);
+  if (e == cudaSuccess && signs_host != nullptr) {
+    e = cudaMalloc(&h->signs, (size_t)h->K_pad);
+    if (e == cudaSuccess) e = cudaMemset(h->signs, 1, (size_t)h->K_pad);
+    if (e == cudaSuccess) e = cudaMemcpy(h->signs, signs_host, (size_t)K, cudaMemcpyHostToDevice);
+  }
   const void* src = W_fp16;
   if (e == cudaSuccess && !w_on_device) {
     e = cudaMalloc(&tmp, (size_t)N * K * 2);
@@ -260,6 +275,7 @@ dptq_status dptq_pack_weights(const void* W_fp16, int N, int K, int had_block, i
   }
   if (e == cudaSuccess) {
     RQArgs a = make_rq(src, N, h->N_pad, K, h->KB, had_block, nfull, tail, log2B, 4, h->sw, h->wt);
+    a.signs = h->signs;
     e = launch_rotate_quant(kRQWeights, a, 0, false);
   }
   if (e == cudaSuccess) e = cudaDeviceSynchronize();
@@ -269,6 +285,52 @@ dptq_status dptq_pack_weights(const void* W_fp16, int N, int K, int had_block, i
     return cuda_fail(e, "dptq_pack_weights");
   }
   *out = h;
+  return DPTQ_OK;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+}  // namespace
+
+dptq_status dptq_pack_weights(const void* W_fp16, int N, int K, int had_block, int w_on_device, dptq_handle* out) {
+  return pack_weights_impl(W_fp16, N, K, had_block, nullptr, w_on_device, out);
+}
+
+dptq_status dptq_pack_weights_rh(const void* W_fp16, int N, int K, int had_block, const int8_t* signs_host,
+                                 int w_on_device, dptq_handle* out) {
+  if (!signs_host) return fail(DPTQ_ERR_INVALID_ARG, "null pointer");
+  return pack_weights_impl(W_fp16, N, K, had_block, signs_host, w_on_device, out);
+}
+
+dptq_status dptq_rotate_quant_act_rh(const void* x_fp16, int M, int K, int had_block, int bits,
+                                     const int8_t* signs_dev, void* codes, float* scales, void* stream) {
+  if (bits != 4 && bits != 8) return fail(DPTQ_ERR_INVALID_ARG, "bits must be 4 or 8");
+  if (M < 0 || K <= 0 || had_block <= 0) return fail(DPTQ_ERR_INVALID_ARG, "bad sizes");
+  if (M == 0) return DPTQ_OK;
+  if (!x_fp16 || !codes || !scales) return fail(DPTQ_ERR_INVALID_ARG, "null pointer");
+  if (signs_dev && !aligned16(signs_dev)) return fail(DPTQ_ERR_INVALID_ARG, "signs must be 16-byte aligned");
+  int nfull, tail, log2B;
+  dptq_status st = check_shape(K, had_block, nfull, tail, log2B);
+  if (st != DPTQ_OK) return st;
+  RQArgs a = make_rq(x_fp16, M, M, K, round_up(K, kKBlock) / kKBlock, had_block, nfull, tail, log2B, bits, scales,
+                     codes);
+  a.signs = signs_dev;
+  DPTQ_CUDA(launch_rotate_quant(kRQPublic, a, static_cast<cudaStream_t>(stream), true), "rotate_quant launch");
+  return DPTQ_OK;
+}
+
+dptq_status dptq_rotate_act_rh(const void* x_fp16, int M, int K, int had_block, const int8_t* signs_dev,
+                               float* y_f32, void* stream) {
+  if (M < 0 || K <= 0 || had_block <= 0) return fail(DPTQ_ERR_INVALID_ARG, "bad sizes");
+  if (M == 0) return DPTQ_OK;
+  if (!x_fp16 || !y_f32) return fail(DPTQ_ERR_INVALID_ARG, "null pointer");
+  if (signs_dev && !aligned16(signs_dev)) return fail(DPTQ_ERR_INVALID_ARG, "signs must be 16-byte aligned");
+  int nfull, tail, log2B;
+  dptq_status st = check_shape(K, had_block, nfull, tail, log2B);
+  if (st != DPTQ_OK) return st;
+  RQArgs a = make_rq(x_fp16, M, M, K, round_up(K, kKBlock) / kKBlock, had_block, nfull, tail, log2B, 4, nullptr,
+                     y_f32);
+  a.signs = signs_dev;
+  DPTQ_CUDA(launch_rotate_quant(kRQY, a, static_cast<cudaStream_t>(stream), true), "rotate launch");
   return DPTQ_OK;
 }
 
@@ -324,6 +386,7 @@ dptq_status quantize_into_scratch(dptq_handle h, const void* x_fp16, int M, int 
   dptq_status st = check_shape(h->K, h->had_block, nfull, tail, log2B);
   if (st != DPTQ_OK) return st;
   RQArgs a = make_rq(x_fp16, M, plan.M_pad, h->K, h->KB, h->had_block, nfull, tail, log2B, bits, sc->sa, sc->act);
+  a.signs = h->signs;
   DPTQ_CUDA(launch_rotate_quant(kRQAct, a, s, true), "rotate_quant launch");
   return DPTQ_OK;
 }
@@ -347,6 +410,7 @@ dptq_status dptq_qlinear(dptq_handle h, const void* x_fp16, int M, int bits, voi
     int nfull, tail, log2B;
     if ((st = check_shape(h->K, h->had_block, nfull, tail, log2B)) != DPTQ_OK) return st;
     fp.args.rq = make_rq(x_fp16, M, fp.M_pad, h->K, h->KB, h->had_block, nfull, tail, log2B, bits, sc->sa, sc->act);
+    fp.args.rq.signs = h->signs;
     return run_gemm(h, fp, sc->act, sc->sa, out_fp16, nullptr, sc, s);
   }
   if ((st = quantize_into_scratch(h, x_fp16, M, bits, plan, sc, s)) != DPTQ_OK) return st;
@@ -401,6 +465,43 @@ dptq_status dptq_qgemm_codes(dptq_handle h, const void* codes, const float* scal
   c.act = sc->act;
   DPTQ_CUDA(launch_codes_to_act(c, s), "codes_to_act launch");
   return run_gemm(h, plan, sc->act, scales, out_fp16, acc_i32, sc, s);
+}
+
+dptq_status dptq_kv4_quantize(const void* kv_fp16, int rows, int cols, int group, void* codes, float* scales,
+                              void* stream) {
+  if (rows < 0 || cols <= 0 || group <= 0) return fail(DPTQ_ERR_INVALID_ARG, "bad sizes");
+  if (rows == 0) return DPTQ_OK;
+  if (!kv_fp16 || !codes || !scales) return fail(DPTQ_ERR_INVALID_ARG, "null pointer");
+  if (!aligned16(kv_fp16)) return fail(DPTQ_ERR_INVALID_ARG, "kv must be 16-byte aligned");
+  if (group % 128 != 0 || group > 1024 || cols % group != 0)
+    return fail(DPTQ_ERR_UNSUPPORTED, "group must be a multiple of 128 up to 1024 that divides cols");
+  int dev;
+  dptq_status st = current_device(&dev);
+  if (st != DPTQ_OK) return st;
+  int sms = 0;
+  DPTQ_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev), "cudaDeviceGetAttribute");
+  KvArgs a{static_cast<const __half*>(kv_fp16), rows, cols, group, static_cast<uint8_t*>(codes), scales};
+  DPTQ_CUDA(launch_kv4(a, sms, static_cast<cudaStream_t>(stream)), "kv4 launch");
+  return DPTQ_OK;
+}
+
+dptq_status dptq_sensitivity_policy(const float* x, const float* dx, int L, int T, int d, int bits, double eps,
+                                    double tau_jr, double tau_snr, double* jr, double* snr, uint8_t* bits_out,
+                                    void* stream) {
+  if (bits != 4 && bits != 8) return fail(DPTQ_ERR_INVALID_ARG, "bits must be 4 or 8");
+  if (L < 0 || T <= 0 || d <= 0 || !(eps >= 0.0)) return fail(DPTQ_ERR_INVALID_ARG, "bad sizes or eps");
+  if (L == 0) return DPTQ_OK;
+  if (!x || !dx || !jr || !snr || !bits_out) return fail(DPTQ_ERR_INVALID_ARG, "null pointer");
+  if (!aligned16(x) || !aligned16(dx) || d % 4 != 0)
+    return fail(DPTQ_ERR_INVALID_ARG, "x and dx must be 16-byte aligned and d a multiple of 4");
+  int dev;
+  dptq_status st = current_device(&dev);
+  if (st != DPTQ_OK) return st;
+  int sms = 0;
+  DPTQ_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev), "cudaDeviceGetAttribute");
+  PolicyArgs a{x, dx, L, T, d, bits, eps, tau_jr, tau_snr, jr, snr, bits_out};
+  DPTQ_CUDA(launch_policy(a, sms, static_cast<cudaStream_t>(stream)), "policy launch");
+  return DPTQ_OK;
 }
 
 dptq_status dptq_reserve(int max_M, int max_K, int max_N) {
@@ -483,6 +584,7 @@ void dptq_destroy(dptq_handle h) {
   if (!h) return;
   if (h->wt) cudaFree(h->wt);
   if (h->sw) cudaFree(h->sw);
+  if (h->signs) cudaFree(h->signs);
   delete h;
 }
 

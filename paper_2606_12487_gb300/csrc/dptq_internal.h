@@ -13,6 +13,7 @@ struct dptq_linear {
   int had_block;
   uint8_t* wt;  // [N_pad/128][KB][4 chunks of 32 k][128 rows][16 B] sign-magnitude nibbles
   float* sw;    // [N_pad]
+  int8_t* signs;  // randomized Hadamard diagonal [K] on the device, or null (plain block Hadamard)
 };
 
 namespace dptq {
@@ -38,6 +39,7 @@ enum RQMode : int {
 
 struct RQArgs {
   const __half* x;   // [rows_in][K] binary16, row-major
+  const int8_t* signs;  // randomized Hadamard diagonal [K] (+1 / -1, 16-byte aligned) or null
   int rows_in;       // rows that carry data (M tokens or N channels)
   int rows_out;      // rows written (padded; rows >= rows_in are zero)
   int K;             // logical K
@@ -70,6 +72,26 @@ struct CodesArgs {
   uint8_t* act;
 };
 cudaError_t launch_codes_to_act(const CodesArgs& a, cudaStream_t s);
+
+// ------------------------------------------------------------------ KV4 and policy
+struct KvArgs {
+  const __half* kv;   // [rows][cols]
+  int rows, cols, group;
+  uint8_t* codes;     // [rows][cols / 2]
+  float* scales;      // [rows][cols / group]
+};
+cudaError_t launch_kv4(const KvArgs& a, int num_sms, cudaStream_t s);
+
+struct PolicyArgs {
+  const float* x;     // [L][T][d]
+  const float* dx;    // [L][T][d]
+  int L, T, d, bits;
+  double eps, tau_jr, tau_snr;
+  double* jr;         // [L]
+  double* snr;        // [L]
+  uint8_t* bits_out;  // [L]
+};
+cudaError_t launch_policy(const PolicyArgs& a, int num_sms, cudaStream_t s);
 
 // ------------------------------------------------------------------ GEMM
 struct GemmArgs {

@@ -125,6 +125,16 @@ __device__ __forceinline__ float ll_to_float_rn(long long S) {
   return S < 0 ? -f : f;
 }
 
+// Randomized Hadamard (QuaRot's diagonal, Sections 1 and 4.2): negate the values whose
+// sign byte is negative (16 consecutive elements; `sg` 16-byte aligned).  Exact.
+__device__ __forceinline__ void apply_signs(const int8_t* sg, long long (&f)[16]) {
+  const uint4 v = *reinterpret_cast<const uint4*>(sg);
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+  for (int e = 0; e < 16; ++e)
+    if ((w[e >> 2] >> (8 * (e & 3) + 7)) & 1u) f[e] = -f[e];
+}
+
 // Correctly rounded fp32 of S * 2^-24 / sqrt(2^log2n) for an exact Hadamard sum S.
 // Even log2n: one rounding of S, then an exact power-of-two scale.  Odd log2n: S and
 // 1/sqrt(2) as fp32 pairs, the product formed with fma to ~2^-47 relative, and one
@@ -205,6 +215,7 @@ __device__ __forceinline__ void rotate_quant_row(const RQArgs& a, int row, unsig
             f[2 * k] = half_to_fixed(w[k] & 0xFFFFu);
             f[2 * k + 1] = half_to_fixed(w[k] >> 16);
           }
+          if (a.signs != nullptr) apply_signs(a.signs + c0 + i0, f);
         } else {
 #pragma unroll
           for (int k = 0; k < 16; ++k) f[k] = 0;
@@ -493,6 +504,7 @@ __device__ __forceinline__ int rq_chunk(const RQArgs& a, const uint4* src, int c
       f[2 * k] = half_to_fixed(w[k] & 0xFFFFu);
       f[2 * k + 1] = half_to_fixed(w[k] >> 16);
     }
+    if (a.signs != nullptr) apply_signs(a.signs + c0 + i0, f);
   } else {
 #pragma unroll
     for (int k = 0; k < 16; ++k) f[k] = 0;

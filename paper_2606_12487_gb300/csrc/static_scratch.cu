@@ -145,6 +145,7 @@ extern "C" dptq_status dptq_qlinear_static(dptq_handle h, const void* x_fp16, in
   a.c_lo = (float)(r2 - (double)a.c_hi);
   a.bits = bits;
   a.scales = sa;
+  a.signs = h->signs;
   a.out = act;
   cudaError_t e = launch_rotate_quant(kRQAct, a, cs, true);
   if (e != cudaSuccess) return static_fail(DPTQ_ERR_CUDA, std::string("rotate_quant launch: ") + cudaGetErrorString(e));

@@ -23,7 +23,9 @@ _STATUS = {0: "ok", 1: "invalid argument", 2: "unsupported shape", 3: "CUDA erro
 EXPORTS = ("dptq_pack_weights", "dptq_rotate_quant_act", "dptq_rotate_act", "dptq_qlinear",
            "dptq_qlinear_quantize", "dptq_qlinear_gemm", "dptq_qlinear_static",
            "dptq_qgemm_codes", "dptq_reserve", "dptq_get_packed", "dptq_get_shape",
-           "dptq_last_device_error", "dptq_destroy", "dptq_status_str", "dptq_last_error_message")
+           "dptq_last_device_error", "dptq_destroy", "dptq_status_str", "dptq_last_error_message",
+           "dptq_pack_weights_rh", "dptq_rotate_quant_act_rh", "dptq_rotate_act_rh", "dptq_kv4_quantize",
+           "dptq_sensitivity_policy")
 
 
 class DptqError(RuntimeError):
@@ -62,6 +64,12 @@ def load(build_if_missing: bool = True):
                 "dptq_destroy": ([P], None),
                 "dptq_status_str": ([I], ctypes.c_char_p),
                 "dptq_last_error_message": ([], ctypes.c_char_p),
+                "dptq_pack_weights_rh": ([P, I, I, I, P, I, ctypes.POINTER(P)], I),
+                "dptq_rotate_quant_act_rh": ([P, I, I, I, I, P, P, P, P], I),
+                "dptq_rotate_act_rh": ([P, I, I, I, P, P, P], I),
+                "dptq_kv4_quantize": ([P, I, I, I, P, P, P], I),
+                "dptq_sensitivity_policy": ([P, P, I, I, I, I, ctypes.c_double, ctypes.c_double, ctypes.c_double,
+                                             P, P, P, P], I),
             }
             for name, (args, res) in sig.items():
                 fn = getattr(lib, name)
@@ -134,6 +142,72 @@ def dptq_pack_weights(W, had_block: int) -> QLinear:
     _check(load().dptq_pack_weights(ctypes.c_void_p(W.data_ptr()), N, K, had_block, int(W.is_cuda),
                                     ctypes.byref(h)))
     return QLinear(h, N, K, had_block)
+
+
+def dptq_pack_weights_rh(W, had_block: int, signs) -> QLinear:
+    """dptq_pack_weights with the randomized Hadamard D R; `signs`: K values of +1 / -1
+    (a host int8 numpy array or CPU tensor)."""
+    import numpy as np
+    import torch
+    if W.dtype != torch.float16 or W.dim() != 2 or not W.is_contiguous():
+        raise TypeError("W must be a contiguous 2-D float16 tensor")
+    N, K = W.shape
+    d = np.ascontiguousarray(signs.cpu().numpy() if isinstance(signs, torch.Tensor) else signs, dtype=np.int8)
+    if d.shape != (K,):
+        raise ValueError(f"signs must have shape ({K},)")
+    h = ctypes.c_void_p()
+    _check(load().dptq_pack_weights_rh(ctypes.c_void_p(W.data_ptr()), N, K, had_block,
+                                       d.ctypes.data_as(ctypes.c_void_p), int(W.is_cuda), ctypes.byref(h)))
+    return QLinear(h, N, K, had_block)
+
+
+def dptq_rotate_quant_act_rh(x, had_block: int, bits: int, signs, codes, scales, stream=None):
+    """dptq_rotate_quant_act with the randomized Hadamard: `signs` a CUDA int8 tensor [K]."""
+    import torch
+    M, K = x.shape
+    _check_tensor(x, torch.float16, (M, K), "x")
+    _check_tensor(signs, torch.int8, (K,), "signs")
+    _check_tensor(codes, torch.uint8 if bits == 4 else torch.int8, (M, K // 2 if bits == 4 else K), "codes")
+    _check_tensor(scales, torch.float32, (M,), "scales")
+    _check(load().dptq_rotate_quant_act_rh(_ptr(x), M, K, had_block, bits, _ptr(signs), _ptr(codes), _ptr(scales),
+                                           _stream(stream)))
+
+
+def dptq_rotate_act_rh(x, had_block: int, signs, y, stream=None):
+    import torch
+    M, K = x.shape
+    _check_tensor(x, torch.float16, (M, K), "x")
+    _check_tensor(signs, torch.int8, (K,), "signs")
+    _check_tensor(y, torch.float32, (M, K), "y")
+    _check(load().dptq_rotate_act_rh(_ptr(x), M, K, had_block, _ptr(signs), _ptr(y), _stream(stream)))
+
+
+def dptq_kv4_quantize(kv, group: int, codes, scales, stream=None):
+    """Group-wise symmetric 4-bit KV codes: kv float16 [rows, cols] -> codes uint8
+    [rows, cols/2] (two's complement nibbles, low nibble first), scales float32
+    [rows, cols/group]."""
+    import torch
+    R, C = kv.shape
+    _check_tensor(kv, torch.float16, (R, C), "kv")
+    _check_tensor(codes, torch.uint8, (R, C // 2), "codes")
+    _check_tensor(scales, torch.float32, (R, C // group if group > 0 else 0), "scales")
+    _check(load().dptq_kv4_quantize(_ptr(kv), R, C, group, _ptr(codes), _ptr(scales), _stream(stream)))
+
+
+def dptq_sensitivity_policy(x, dx, bits: int, eps: float, tau_jr: float, tau_snr: float, jr, snr, bits_out,
+                            stream=None):
+    """Per-layer JR and historical SNR of residual states x and updates dx (float32
+    [L, T, d]) and the activation bits (8 on the sensitive set): jr, snr float64 [L],
+    bits_out uint8 [L]."""
+    import torch
+    L, T, d = x.shape
+    _check_tensor(x, torch.float32, (L, T, d), "x")
+    _check_tensor(dx, torch.float32, (L, T, d), "dx")
+    _check_tensor(jr, torch.float64, (L,), "jr")
+    _check_tensor(snr, torch.float64, (L,), "snr")
+    _check_tensor(bits_out, torch.uint8, (L,), "bits_out")
+    _check(load().dptq_sensitivity_policy(_ptr(x), _ptr(dx), L, T, d, bits, eps, tau_jr, tau_snr, _ptr(jr), _ptr(snr),
+                                          _ptr(bits_out), _stream(stream)))
 
 
 def dptq_rotate_quant_act(x, had_block: int, bits: int, codes, scales, stream=None):

@@ -78,3 +78,26 @@ def test_binding_has_no_cpu_fallback():
     assert "import oracle" not in src and "from oracle" not in src
     for banned in ("numpy.matmul", "torch.matmul", "@ ", "hadamard"):
         assert banned not in src
+
+
+def test_next_entry_points_check_arguments_without_gpu(lib):
+    P = ctypes.c_void_p
+    dummy = P(16)
+    h = P()
+    # randomized Hadamard packing: null signs
+    assert lib.dptq_pack_weights_rh(dummy, 16, 256, 256, None, 1, ctypes.byref(h)) == 1
+    # misaligned device signs
+    assert lib.dptq_rotate_quant_act_rh(dummy, 4, 256, 256, 4, P(17), dummy, dummy, None) == 1
+    assert lib.dptq_rotate_act_rh(dummy, 4, 256, 256, P(18), dummy, None) == 1
+    # KV4: null pointers, group not a multiple of 128 / not dividing cols, rows == 0
+    assert lib.dptq_kv4_quantize(None, 4, 256, 128, dummy, dummy, None) == 1
+    assert lib.dptq_kv4_quantize(dummy, 4, 256, 100, dummy, dummy, None) == 2
+    assert lib.dptq_kv4_quantize(dummy, 4, 384, 256, dummy, dummy, None) == 2
+    assert lib.dptq_kv4_quantize(dummy, 0, 256, 128, dummy, dummy, None) == 0
+    # policy: bits, eps, sizes, null pointers, L == 0
+    D = ctypes.c_double
+    assert lib.dptq_sensitivity_policy(dummy, dummy, 2, 8, 64, 5, D(1e-6), D(0.1), D(20.0), dummy, dummy, dummy, None) == 1
+    assert lib.dptq_sensitivity_policy(dummy, dummy, 2, 8, 64, 4, D(-1.0), D(0.1), D(20.0), dummy, dummy, dummy, None) == 1
+    assert lib.dptq_sensitivity_policy(dummy, dummy, 2, 8, 63, 4, D(1e-6), D(0.1), D(20.0), dummy, dummy, dummy, None) == 1
+    assert lib.dptq_sensitivity_policy(None, dummy, 2, 8, 64, 4, D(1e-6), D(0.1), D(20.0), dummy, dummy, dummy, None) == 1
+    assert lib.dptq_sensitivity_policy(dummy, dummy, 0, 8, 64, 4, D(1e-6), D(0.1), D(20.0), dummy, dummy, dummy, None) == 0
