@@ -405,7 +405,7 @@ def run_shapes(args):
         return e0.elapsed_time(e1) * 1e3 / reps
 
     rows = []
-    for label, M, N, K, B, bits in shape_cases():
+    for label, M, N, K, B, bits in ([] if args.extra_only else shape_cases()):
         wbytes = N * K // 2
         copies = max(1, min(64, math.ceil(2 * L2_BYTES / wbytes)))
         W = inputs.torch_weights(N, K, 0, 0, dev)
@@ -594,6 +594,8 @@ def main(argv=None):
                     help="run only the first L layers (small cases for profiler captures; 0 = all)")
     ap.add_argument("--shapes", action="store_true",
                     help="time each decode / prefill projection shape alone and print one JSON line of them")
+    ap.add_argument("--extra-only", action="store_true",
+                    help="with --shapes: time only the KV4 quantizer and the sensitivity policy")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         args.warmup = 3

@@ -113,8 +113,8 @@ dptq_status dptq_rotate_quant_act_rh(const void* x_fp16, int M, int K, int had_b
 dptq_status dptq_rotate_act_rh(const void* x_fp16, int M, int K, int had_block, const int8_t* signs_dev,
                                float* y_f32, void* stream);
 
-/* KV-cache quantization (Section 4.2: "group-wise quantization with a group size of
- * 128", 4 bits).  kv_fp16: device [rows][cols] binary16 (16-byte aligned).  Each row is
+/* KV-cache quantization (Section 4.2: 4-bit KV cache, quantized in groups of 128
+ * values).  kv_fp16: device [rows][cols] binary16 (16-byte aligned).  Each row is
  * cut into groups of `group` consecutive columns, each quantized on its own,
  * symmetrically (the paper does not say symmetric or asymmetric): s = max|x| / 7 in
  * fp32 (IEEE division), c = clamp(round-half-even(x / s), -8, 7) (never -8), an
@@ -138,7 +138,13 @@ dptq_status dptq_kv4_quantize(const void* kv_fp16, int rows, int cols, int group
  * x, dx: device fp32 [L][T][d], 16-byte aligned, d % 4 == 0; jr, snr: device double
  * [L] (written); bits_out: device uint8 [L] (written).  bits in {4, 8}; eps >= 0 (the
  * paper's epsilon; its value is not given).  Norms and errors are evaluated in fp32 per
- * element and summed in fp64 per token.  Asynchronous. */
+ * element and summed per token (in fp32 for d <= 4096: sums of non-negative terms, a
+ * relative error below 2^-19) and the per-layer means accumulate in fp64: JR within
+ * 1e-5 relative and SNR within 1e-3 dB of the exact statistics.  Asynchronous.  INVALID_ARG for bad sizes, bits, eps, null or misaligned pointers.  The
+ * first call on a device allocates the library's small per-device scratch (its error
+ * word), which is refused (UNSUPPORTED) during stream capture: call dptq_reserve first.
+ * A bounded in-kernel wait that gave up leaves jr/snr unspecified and is reported by
+ * dptq_last_device_error (TIMEOUT). */
 dptq_status dptq_sensitivity_policy(const float* x, const float* dx, int L, int T, int d, int bits, double eps,
                                     double tau_jr, double tau_snr, double* jr, double* snr, uint8_t* bits_out,
                                     void* stream);

@@ -497,10 +497,11 @@ dptq_status dptq_sensitivity_policy(const float* x, const float* dx, int L, int 
   int dev;
   dptq_status st = current_device(&dev);
   if (st != DPTQ_OK) return st;
-  int sms = 0;
-  DPTQ_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev), "cudaDeviceGetAttribute");
-  PolicyArgs a{x, dx, L, T, d, bits, eps, tau_jr, tau_snr, jr, snr, bits_out};
-  DPTQ_CUDA(launch_policy(a, sms, static_cast<cudaStream_t>(stream)), "policy launch");
+  Scratch* sc = nullptr;
+  st = ensure_scratch(dev, 0, 0, static_cast<cudaStream_t>(stream), &sc);
+  if (st != DPTQ_OK) return st;
+  PolicyArgs a{x, dx, L, T, d, bits, eps, tau_jr, tau_snr, jr, snr, bits_out, sc->err};
+  DPTQ_CUDA(launch_policy(a, sc->num_sms, static_cast<cudaStream_t>(stream)), "policy launch");
   return DPTQ_OK;
 }
 

@@ -90,6 +90,7 @@ struct PolicyArgs {
   double* jr;         // [L]
   double* snr;        // [L]
   uint8_t* bits_out;  // [L]
+  int* err;           // device error word (bounded waits that gave up)
 };
 cudaError_t launch_policy(const PolicyArgs& a, int num_sms, cudaStream_t s);
 

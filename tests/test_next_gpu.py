@@ -98,8 +98,9 @@ def test_randomized_pack_rejects_bad_signs(dp):
 
 
 # ---------------------------------------------------------------- KV4
+# (5, 384): 15 groups of 128, a ragged last set of four for the group-128 kernel
 @pytest.mark.parametrize("rows,cols,group", [(1, 128, 128), (37, 1024, 128), (64, 4096, 128), (9, 2048, 256),
-                                             (3, 3072, 1024)])
+                                             (3, 3072, 1024), (5, 384, 128)])
 def test_kv4_bit_exact(dp, orc, rows, cols, group):
     rng = np.random.default_rng(rows * cols + group)
     x = (rng.standard_normal((rows, cols)) * np.float32(4.0) ** rng.integers(-4, 4, (rows, 1))).astype(np.float32)
@@ -107,6 +108,11 @@ def test_kv4_bit_exact(dp, orc, rows, cols, group):
     if rows > 2:
         x[2, 5] = 65504.0                                  # fp16 maximum
         x[1, group:2 * group] = np.float32(1e-6) * rng.standard_normal(group).astype(np.float32)   # subnormal range
+    if rows > 3:
+        # a group with s = 1 exactly and x / s on half-integers: every code is a tie
+        # (round half to even), e.g. 0.5 -> 0, 1.5 -> 2, -2.5 -> -2
+        x[3, :group] = (rng.integers(-7, 7, group) + np.float32(0.5)).astype(np.float32)
+        x[3, 0] = 7.0
     xh = inputs.to_f16(x)
     kv = torch.from_numpy(xh).to(DEV)
     codes = torch.empty((rows, cols // 2), dtype=torch.uint8, device=DEV)
@@ -148,7 +154,11 @@ def _residual_streams(L, T, d, seed):
     return x, dx
 
 
-@pytest.mark.parametrize("L,T,d,bits", [(6, 16, 256, 4), (4, 8, 4096, 4), (3, 5, 1000, 8)])
+# Small cases (one token per CTA), ranges of several tokens per CTA that wrap the
+# kernel's ring of token stages and cross layer boundaries (8 x 300 and 4 x 300 tokens),
+# and a token wider than 4096 (the unstaged kernel).
+@pytest.mark.parametrize("L,T,d,bits", [(6, 16, 256, 4), (4, 8, 4096, 4), (3, 5, 1000, 8),
+                                        (8, 300, 512, 4), (4, 300, 4096, 8), (3, 7, 5120, 4)])
 def test_policy_stats_and_mask(dp, orc, L, T, d, bits):
     x, dx = _residual_streams(L, T, d, L * T + d)
     jr_ref = np.empty(L)
