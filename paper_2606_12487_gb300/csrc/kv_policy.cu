@@ -44,8 +44,8 @@ __device__ __forceinline__ float absmax4(uint2 raw) {
                fmaxf(fabsf(__low2float(h1)), fabsf(__high2float(h1))));
 }
 
-// Groups of 128 (the paper's size): four consecutive groups per warp and iteration, all
-// four loads issued first, so that each SM keeps enough bytes in flight.
+// Groups of 128 (the paper's size): kKvQuads sets of four consecutive groups per warp and
+// iteration, all loads issued first, so that each SM keeps enough bytes in flight.
 //   * The four groups' maxima are reduced by one transposed butterfly (6 exchanges, not
 //     20): afterwards lane l holds the maximum of group 2 (l >> 4) + ((l >> 3) & 1), so
 //     every lane forms one scale and reciprocal and lanes 0, 8, 16, 24 hand them out.
@@ -55,57 +55,65 @@ __device__ __forceinline__ float absmax4(uint2 raw) {
 //     of a half-integer, the IEEE quotient y / s decides instead (|y r - y / s| and
 //     |fl(y / s) - y / s| are both below 2^-21, so elsewhere the two agree).
 constexpr float kRoundMagic = 12582912.0f;   // 1.5 * 2^23
+constexpr int kKvQuads = 2;
 
 __global__ void __launch_bounds__(kKvWarps * 32) kv4_quantize_g128_kernel(const KvArgs a) {
   const int lane = threadIdx.x & 31;
   const int my_g = ((lane >> 4) << 1) | ((lane >> 3) & 1);
   const bool up16 = (lane & 16) != 0, up8 = (lane & 8) != 0;
   const long long ngroups = (long long)a.rows * (a.cols >> 7);   // groups are consecutive in memory
-  const long long nquads = (ngroups + 3) >> 2;
+  const long long nitems = (ngroups + 4 * kKvQuads - 1) / (4 * kKvQuads);
   const long long nwarps = (long long)gridDim.x * kKvWarps;
-  for (long long w = (long long)blockIdx.x * kKvWarps + (threadIdx.x >> 5); w < nquads; w += nwarps) {
-    const long long g0 = 4 * w;
-    const int ng = ngroups - g0 < 4 ? (int)(ngroups - g0) : 4;
-    uint2 raw[4];
+  for (long long w = (long long)blockIdx.x * kKvWarps + (threadIdx.x >> 5); w < nitems; w += nwarps) {
+    uint2 raws[4 * kKvQuads];
 #pragma unroll
-    for (int i = 0; i < 4; ++i)
-      raw[i] = i < ng ? __ldg(reinterpret_cast<const uint2*>(a.kv + (size_t)(g0 + i) * 128 + 4 * lane))
-                      : make_uint2(0u, 0u);
-    float m[4];
+    for (int i = 0; i < 4 * kKvQuads; ++i) {
+      const long long g = 4 * kKvQuads * w + i;
+      raws[i] = g < ngroups ? __ldg(reinterpret_cast<const uint2*>(a.kv + (size_t)g * 128 + 4 * lane))
+                            : make_uint2(0u, 0u);
+    }
 #pragma unroll
-    for (int i = 0; i < 4; ++i) m[i] = absmax4(raw[i]);
-    float k0 = up16 ? m[2] : m[0], k1 = up16 ? m[3] : m[1];
-    k0 = fmaxf(k0, __shfl_xor_sync(0xffffffffu, up16 ? m[0] : m[2], 16));
-    k1 = fmaxf(k1, __shfl_xor_sync(0xffffffffu, up16 ? m[1] : m[3], 16));
-    float amax = fmaxf(up8 ? k1 : k0, __shfl_xor_sync(0xffffffffu, up8 ? k0 : k1, 8));
+    for (int q = 0; q < kKvQuads; ++q) {
+      const long long g0 = 4 * kKvQuads * w + 4 * q;
+      if (g0 >= ngroups) break;
+      const int ng = ngroups - g0 < 4 ? (int)(ngroups - g0) : 4;
+      const uint2* raw = raws + 4 * q;
+      float m[4];
 #pragma unroll
-    for (int o = 4; o > 0; o >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, o));
-    const float s_mine = __fdiv_rn(amax, 7.f);   // 0 for an all-zero group
-    const float r_mine = amax > 0.f ? __frcp_rn(s_mine) : 0.f;
-    if ((lane & 7) == 0 && my_g < ng) a.scales[g0 + my_g] = s_mine;
+      for (int i = 0; i < 4; ++i) m[i] = absmax4(raw[i]);
+      float k0 = up16 ? m[2] : m[0], k1 = up16 ? m[3] : m[1];
+      k0 = fmaxf(k0, __shfl_xor_sync(0xffffffffu, up16 ? m[0] : m[2], 16));
+      k1 = fmaxf(k1, __shfl_xor_sync(0xffffffffu, up16 ? m[1] : m[3], 16));
+      float amax = fmaxf(up8 ? k1 : k0, __shfl_xor_sync(0xffffffffu, up8 ? k0 : k1, 8));
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const float s = __shfl_sync(0xffffffffu, s_mine, 8 * i);
-      const float r = __shfl_sync(0xffffffffu, r_mine, 8 * i);
-      const __half2 h0 = *reinterpret_cast<const __half2*>(&raw[i].x);
-      const __half2 h1 = *reinterpret_cast<const __half2*>(&raw[i].y);
-      const float y[4] = {__low2float(h0), __high2float(h0), __low2float(h1), __high2float(h1)};
-      float tb[4];
-      uint32_t nearm = 0;
+      for (int o = 4; o > 0; o >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, o));
+      const float s_mine = __fdiv_rn(amax, 7.f);   // 0 for an all-zero group
+      const float r_mine = amax > 0.f ? __frcp_rn(s_mine) : 0.f;
+      if ((lane & 7) == 0 && my_g < ng) a.scales[g0 + my_g] = s_mine;
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        tb[e] = __fmaf_rn(y[e], r, kRoundMagic);
-        const float f = __fmaf_rn(y[e], r, -__fsub_rn(tb[e], kRoundMagic));
-        nearm |= fabsf(f) >= 0.5f - 0x1p-15f ? (1u << e) : 0u;
+      for (int i = 0; i < 4; ++i) {
+        const float s = __shfl_sync(0xffffffffu, s_mine, 8 * i);
+        const float r = __shfl_sync(0xffffffffu, r_mine, 8 * i);
+        const __half2 h0 = *reinterpret_cast<const __half2*>(&raw[i].x);
+        const __half2 h1 = *reinterpret_cast<const __half2*>(&raw[i].y);
+        const float y[4] = {__low2float(h0), __high2float(h0), __low2float(h1), __high2float(h1)};
+        float tb[4];
+        uint32_t nearm = 0;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          tb[e] = __fmaf_rn(y[e], r, kRoundMagic);
+          const float f = __fmaf_rn(y[e], r, -__fsub_rn(tb[e], kRoundMagic));
+          nearm |= fabsf(f) >= 0.5f - 0x1p-15f ? (1u << e) : 0u;
+        }
+        if (__any_sync(0xffffffffu, nearm != 0u)) {
+#pragma unroll
+          for (int e = 0; e < 4; ++e)
+            if ((nearm >> e) & 1u) tb[e] = __fadd_rn(rintf(__fdiv_rn(y[e], s)), kRoundMagic);
+        }
+        const uint32_t packed = (__float_as_uint(tb[0]) & 0xFu) | ((__float_as_uint(tb[1]) & 0xFu) << 4) |
+                                ((__float_as_uint(tb[2]) & 0xFu) << 8) | ((__float_as_uint(tb[3]) & 0xFu) << 12);
+        if (i < ng) reinterpret_cast<uint16_t*>(a.codes + (size_t)(g0 + i) * 64)[lane] = (uint16_t)packed;
       }
-      if (__any_sync(0xffffffffu, nearm != 0u)) {
-#pragma unroll
-        for (int e = 0; e < 4; ++e)
-          if ((nearm >> e) & 1u) tb[e] = __fadd_rn(rintf(__fdiv_rn(y[e], s)), kRoundMagic);
-      }
-      const uint32_t packed = (__float_as_uint(tb[0]) & 0xFu) | ((__float_as_uint(tb[1]) & 0xFu) << 4) |
-                              ((__float_as_uint(tb[2]) & 0xFu) << 8) | ((__float_as_uint(tb[3]) & 0xFu) << 12);
-      if (i < ng) reinterpret_cast<uint16_t*>(a.codes + (size_t)(g0 + i) * 64)[lane] = (uint16_t)packed;
     }
   }
 }
@@ -159,9 +167,16 @@ __global__ void __launch_bounds__(kKvWarps * 32) kv4_quantize_kernel(const KvArg
 
 cudaError_t launch_kv4(const KvArgs& a, int num_sms, cudaStream_t s) {
   const long long ngroups = (long long)a.rows * (a.cols / a.group);
-  const long long work = a.group == 128 ? (ngroups + 3) / 4 : ngroups;   // warps' work items
+  const long long work = a.group == 128 ? (ngroups + 4 * kKvQuads - 1) / (4 * kKvQuads) : ngroups;   // warps' items
   long long blocks = (work + kKvWarps - 1) / kKvWarps;
-  const long long cap = (long long)num_sms * 8;
+  int per_sm = 8;
+  if (a.group == 128) {   // one wave of resident CTAs
+    const cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kv4_quantize_g128_kernel,
+                                                                        kKvWarps * 32, 0);
+    if (e != cudaSuccess) return e;
+    if (per_sm < 1) per_sm = 1;
+  }
+  const long long cap = (long long)num_sms * per_sm;
   if (blocks > cap) blocks = cap;
   if (blocks < 1) blocks = 1;
   if (a.group == 128)

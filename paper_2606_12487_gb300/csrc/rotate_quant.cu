@@ -12,8 +12,11 @@
 
 namespace dptq {
 
+// Three CTAs per SM (at most 85 registers a thread; the body needs 72 without spilling):
+// many-row launches (prefill) are bound by the latency of each row's chain of steps, so
+// rows in flight per SM set their throughput.
 template <int MODE>
-__global__ void __launch_bounds__(kRQThreads) rotate_quant_kernel(const RQArgs a) {
+__global__ void __launch_bounds__(kRQThreads, 3) rotate_quant_kernel(const RQArgs a) {
   extern __shared__ __align__(16) unsigned char rq_smem[];
   __shared__ float red[kRQThreads / 32];
   pdl_launch_dependents();
