@@ -406,6 +406,8 @@ def run_shapes(args):
 
     rows = []
     for label, M, N, K, B, bits in ([] if args.extra_only else shape_cases()):
+        if args.only and args.only not in f"{label} M={M} A{bits}":
+            continue
         wbytes = N * K // 2
         copies = max(1, min(64, math.ceil(2 * L2_BYTES / wbytes)))
         W = inputs.torch_weights(N, K, 0, 0, dev)
@@ -596,6 +598,9 @@ def main(argv=None):
                     help="time each decode / prefill projection shape alone and print one JSON line of them")
     ap.add_argument("--extra-only", action="store_true",
                     help="with --shapes: time only the KV4 quantizer and the sensitivity policy")
+    ap.add_argument("--only", default="",
+                    help="with --shapes: only the shapes whose label 'NAME M=.. A..' contains this text "
+                         "(the KV4 and policy timings still follow)")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         args.warmup = 3

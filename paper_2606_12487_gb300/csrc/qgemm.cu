@@ -557,8 +557,13 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
       const int mt = un.tile - nt * a.m_tiles;
       const int n = nt * 128 + q * 32 + lane;
       const int m0 = mt * NT;
-      // Scales are fetched while the MMAs of this unit still run.
+      // Scales are fetched while the MMAs of this unit still run.  Tiles of more than 64
+      // tokens take their token scales 32 at a time, one per lane (coalesced), and hand
+      // them out by shuffles.
       const float swn = n < a.N ? sw_g[n] : 0.f;
+      auto sa_group = [&](int c) { return m0 + c + lane < a.M ? __ldg(sa_g + m0 + c + lane) : 0.f; };
+      float sa_nxt = NT > 64 ? sa_group(0) : 0.f;
+      float sa_grp = 0.f;
       if (NT <= 64 && mt != sa_mt) {
         if (!epi_sync()) break;   // every warp is done with the previous token tile's scales
         for (int i = etid; i < NT; i += kNumEpiWarps * 32) sa_sh[i] = m0 + i < a.M ? sa_g[m0 + i] : 0.f;
@@ -591,8 +596,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
         __half hv[16];
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
-          const int m = m0 + c0 + i;
-          const float sav = NT <= 64 ? sa_sh[c0 + i] : (m < a.M ? __ldg(sa_g + m) : 0.f);
+          const float sav = NT <= 64 ? sa_sh[c0 + i] : __shfl_sync(0xffffffffu, sa_grp, (c0 & 31) + i);
           hv[i] = __float2half_rn(__fmul_rn(__fmul_rn(__int2float_rn(v[i]), sav), swn));
         }
         if (acc_g != nullptr && n < a.N) {
@@ -627,44 +631,69 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
       // access covers 512 contiguous bytes); otherwise int32 atomics, token-major.
       const bool f32 = a.segs == 1;
       float* const wslf = wsl != nullptr ? reinterpret_cast<float*>(wsl) + (size_t)(q * 32 + lane) * 4 : nullptr;
-#pragma unroll 1
-      for (int c0 = 0; c0 < NT; c0 += 16) {
-        int acc[16];
-        if (f32) {
-          float f[16];
-          if (finish && wsl != nullptr) {
+      if (f32) {
+        // Chunks of 16 tokens, two per iteration.  When this CTA finishes a split tile, the
+        // slot reads of the next chunk are issued before the current chunk is processed,
+        // so their L2 latency overlaps that work.
+        const bool rd = finish && wsl != nullptr;
+        float4 s0[4], s1[4];
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-              const float4 t = __ldcg(reinterpret_cast<const float4*>(wslf + (c0 / 4 + j) * 512));
-              f[4 * j] = t.x;
-              f[4 * j + 1] = t.y;
-              f[4 * j + 2] = t.z;
-              f[4 * j + 3] = t.w;
-            }
+        for (int j = 0; j < 4; ++j) s0[j] = s1[j] = make_float4(0.f, 0.f, 0.f, 0.f);
+        auto load_slot = [&](int c, float4 (&d)[4]) {
+#pragma unroll
+          for (int j = 0; j < 4; ++j) d[j] = __ldcg(reinterpret_cast<const float4*>(wslf + (c / 4 + j) * 512));
+        };
+        auto chunk = [&](int c, const float4 (&sv)[4]) {
+          uint32_t r[16];
+          tmem_ld16(tb + (uint32_t)c, r);
+          tmem_ld_wait();
+          if (etid == 0 && c == 0) DPTQ_TRACE_POINT(tr, 2);
+          float f[16];
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            f[4 * j] = __fadd_rn(sv[j].x, __uint_as_float(r[4 * j]));
+            f[4 * j + 1] = __fadd_rn(sv[j].y, __uint_as_float(r[4 * j + 1]));
+            f[4 * j + 2] = __fadd_rn(sv[j].z, __uint_as_float(r[4 * j + 2]));
+            f[4 * j + 3] = __fadd_rn(sv[j].w, __uint_as_float(r[4 * j + 3]));
+          }
+          if (rd) {
 #pragma unroll
             for (int j = 0; j < 4; ++j)   // zero for the next launch
-              __stcg(reinterpret_cast<float4*>(wslf + (c0 / 4 + j) * 512), make_float4(0.f, 0.f, 0.f, 0.f));
-          } else {
-#pragma unroll
-            for (int i = 0; i < 16; ++i) f[i] = 0.f;
+              __stcg(reinterpret_cast<float4*>(wslf + (c / 4 + j) * 512), make_float4(0.f, 0.f, 0.f, 0.f));
           }
-          uint32_t r[16];
-          tmem_ld16(tb + (uint32_t)c0, r);
-          tmem_ld_wait();
-          if (etid == 0 && c0 == 0) DPTQ_TRACE_POINT(tr, 2);
-#pragma unroll
-          for (int i = 0; i < 16; ++i) f[i] = __fadd_rn(f[i], __uint_as_float(r[i]));
-          if (etid == 0) DPTQ_TRACE_POINT(tr, c0 == 0 ? 4 : 119);
+          if (etid == 0) DPTQ_TRACE_POINT(tr, c == 0 ? 4 : 119);
           if (finish) {
+            int acc[16];
 #pragma unroll
             for (int i = 0; i < 16; ++i) acc[i] = __float2int_rn(f[i] * 512.f);
-            write_out(c0, acc);
+            write_out(c, acc);
           } else {
 #pragma unroll
             for (int j = 0; j < 4; ++j)
-              red_add_v4_f32(wslf + (c0 / 4 + j) * 512, f[4 * j], f[4 * j + 1], f[4 * j + 2], f[4 * j + 3]);
+              red_add_v4_f32(wslf + (c / 4 + j) * 512, f[4 * j], f[4 * j + 1], f[4 * j + 2], f[4 * j + 3]);
           }
-        } else {
+          if (etid == 0) DPTQ_TRACE_POINT(tr, c == 0 ? 6 : 123);
+        };
+        if (rd) load_slot(0, s0);
+#pragma unroll 1
+        for (int c0 = 0; c0 < NT; c0 += 32) {
+          if (NT > 64) {
+            sa_grp = sa_nxt;
+            if (c0 + 32 < NT) sa_nxt = sa_group(c0 + 32);
+          }
+          const bool two = c0 + 16 < NT;
+          if (rd && two) load_slot(c0 + 16, s1);
+          chunk(c0, s0);
+          if (two) {
+            if (rd && c0 + 32 < NT) load_slot(c0 + 32, s0);
+            chunk(c0 + 16, s1);
+          }
+        }
+      } else {
+#pragma unroll 1
+        for (int c0 = 0; c0 < NT; c0 += 16) {
+          int acc[16];
+          if (NT > 64 && (c0 & 31) == 0) sa_grp = sa_group(c0);
           if (finish && wsl != nullptr) {
 #pragma unroll
             for (int i = 0; i < 16; ++i) acc[i] = __ldcg(wsl + (c0 + i) * 128 + q * 32 + lane);
@@ -687,8 +716,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
 #pragma unroll
             for (int i = 0; i < 16; ++i) atomicAdd(wsl + (c0 + i) * 128 + q * 32 + lane, acc[i]);
           }
+          if (etid == 0) DPTQ_TRACE_POINT(tr, c0 == 0 ? 6 : 123);
         }
-        if (etid == 0) DPTQ_TRACE_POINT(tr, c0 == 0 ? 6 : 123);
       }
       if (etid == 0 && u < 4) DPTQ_TRACE_POINT(tr, 112 + u);
       tc_fence_before();
@@ -713,6 +742,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
 #pragma unroll 1
           for (int c0 = 0; c0 < NT; c0 += 16) {
             int v[16];
+            if (NT > 64 && (c0 & 31) == 0) sa_grp = sa_group(c0);
             if (f32) {
 #pragma unroll
               for (int j = 0; j < 4; ++j) {
