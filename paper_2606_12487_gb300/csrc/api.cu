@@ -3,6 +3,7 @@
 // every step of the path runs in the kernels of rotate_quant.cu and qgemm.cu.
 #include <cmath>
 #include <cstdint>
+#include <algorithm>
 #include <cstdio>
 #include <cstdlib>
 #include <cstring>
@@ -511,7 +512,9 @@ dptq_status dptq_reserve(int max_M, int max_K, int max_N) {
   dptq_status st = current_device(&dev);
   if (st != DPTQ_OK) return st;
   (void)max_N;
-  const size_t M_pad = (size_t)round_up(max_M > 0 ? max_M : 1, kMaxNT);
+  // Rows of the widest token tile and of the 192-token prefill tile.
+  const int m_res = max_M > 0 ? max_M : 1;
+  const size_t M_pad = (size_t)std::max(round_up(m_res, kMaxNT), round_up(m_res, 192));
   const size_t K_pad = (size_t)round_up(max_K > 0 ? max_K : kKBlock, kKBlock);
   Scratch* sc = nullptr;
   st = ensure_scratch(dev, 2 * K_pad * M_pad, M_pad, 0, &sc);

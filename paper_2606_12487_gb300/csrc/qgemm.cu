@@ -128,6 +128,12 @@ __device__ __forceinline__ uint32_t widen_hi(uint32_t w) {
   return ((w >> 4) & 0x07070707u) | (w & 0x80808080u);
 }
 
+// Where the widened weights (the MMA's A operand) live: tensor memory for two-block
+// stages (decode) and for 192-token tiles, whose two accumulators (384 columns) leave
+// 128 columns for four one-block slots; shared memory otherwise.  With the A operand in
+// tensor memory a stage costs shared memory only its bulk copies and the MMA's B reads.
+__host__ __device__ constexpr bool a_in_tmem(int nt, int kps) { return kps == 2 || nt == 192; }
+
 // Shared-memory layout: a ring of `conv_slots` widened weight slots (KPS tiles of 16 KB
 // each, 1024-aligned swizzle atoms; absent when the widened weights live in tensor
 // memory) followed by the `stages`-deep ring of bulk-copy slots.  A bulk-copy slot holds
@@ -158,10 +164,10 @@ struct Smem {
 // scales after the same point.  The last CTA to finish resets the counters.
 template <int NT, int KPS, bool FUSED>
 __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a) {
-  // Two-block stages (token tiles of up to 64, weight streaming) widen the weights
-  // straight into tensor memory and feed the MMA's A operand from there; one-block
-  // stages widen into shared memory.
-  constexpr bool kATmem = (KPS == 2);
+  // Two-block stages (token tiles of up to 64, weight streaming) and 192-token tiles
+  // widen the weights straight into tensor memory and feed the MMA's A operand from
+  // there; other one-block stages widen into shared memory.
+  constexpr bool kATmem = a_in_tmem(NT, KPS);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int S = a.stages;
@@ -296,11 +302,13 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
       const uint8_t* asrc = a.act + ((size_t)un.i0 * KPS * a.M_pad + (size_t)mt * NT) * 128;
       for (int it = un.i0; it < un.i1; ++it, ++g, rg.next(), wsrc += w_bytes, asrc += KPS * kb_stride) {
         const int s = rg.s;
+        if (leader && g == 8) DPTQ_TRACE_CLOCK(tr, 242);
         if (!mbar_wait_warp(&empty[s], rg.ph ^ 1u, abort_flag, a.err, kDevTimeoutEmpty)) {
           ok = false;
           break;
         }
         if (leader) {
+          if (g == 8) DPTQ_TRACE_CLOCK(tr, 241);
           if (g < 16) DPTQ_TRACE_POINT(tr, 8 + g);
           mbar_arrive_expect_tx(&full[s], w_bytes);
           bulk_g2s(sm.wpack(s), wsrc, w_bytes, &full[s], pol_w);
@@ -372,12 +380,18 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
       bool ok = true;
       for (int it = un.i0; it < un.i1; ++it, rg.next(), rc.next()) {
         const int s = rg.s, c = rc.s;
-        if (!mbar_wait_warp(&afull[s], rg.ph, abort_flag, a.err, kDevTimeoutFull) ||
-            !mbar_wait_warp(&cfull[c], rc.ph, abort_flag, a.err, kDevTimeoutConv)) {
+        if (leader && it - un.i0 + mma_done == 8) DPTQ_TRACE_CLOCK(tr, 237);
+        if (!mbar_wait_warp(&afull[s], rg.ph, abort_flag, a.err, kDevTimeoutFull)) {
+          ok = false;
+          break;
+        }
+        if (leader && it - un.i0 + mma_done == 8) DPTQ_TRACE_CLOCK(tr, 239);
+        if (!mbar_wait_warp(&cfull[c], rc.ph, abort_flag, a.err, kDevTimeoutConv)) {
           ok = false;
           break;
         }
         const int gm = it - un.i0 + mma_done;
+        if (leader && gm == 8) DPTQ_TRACE_CLOCK(tr, 235);
         if (leader && gm < 16) DPTQ_TRACE_POINT(tr, 72 + gm);
         tc_fence_after();
         if (seg_left == 0) {   // next exact-accumulation segment: next accumulator
@@ -408,6 +422,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
           }
           mma_commit(&empty[s]);
           mma_commit(&cempty[c]);
+          if (gm == 8) DPTQ_TRACE_CLOCK(tr, 236);
           if (gm < 16) DPTQ_TRACE_POINT(tr, 88 + gm);
         }
         __syncwarp();
@@ -460,15 +475,46 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
       bool ok = true;
       for (int it = un.i0; it < un.i1; ++it, rg.next(), rc.next()) {
         const int s = rg.s, c = rc.s;
-        if (!mbar_wait(&full[s], rg.ph, abort_flag, a.err, kDevTimeoutFull) ||
-            !mbar_wait(&cempty[c], rc.ph ^ 1u, abort_flag, a.err, kDevTimeoutConv)) {
+        if (ctid == 0 && it - un.i0 + cvt_done == 8) DPTQ_TRACE_CLOCK(tr, 238);
+        if (!mbar_wait(&full[s], rg.ph, abort_flag, a.err, kDevTimeoutFull)) {
+          ok = false;
+          break;
+        }
+        if (ctid == 0 && it - un.i0 + cvt_done == 8) DPTQ_TRACE_CLOCK(tr, 240);
+        if (!mbar_wait(&cempty[c], rc.ph ^ 1u, abort_flag, a.err, kDevTimeoutConv)) {
           ok = false;
           break;
         }
         const int gc = it - un.i0 + cvt_done;
         if (ctid == 0 && gc < 16) DPTQ_TRACE_POINT(tr, 40 + gc);
         const uint8_t* __restrict__ wp = sm.wpack(s);
-        if constexpr (kATmem) {
+        if constexpr (kATmem && KPS == 1) {
+          // Warp (lane quarter q, half hs) widens k columns 64 hs .. 64 hs + 63 of rows
+          // 32q..32q+31: each thread reads its row's 32 packed bytes (chunks 2 hs and
+          // 2 hs + 1 of 32 k) and stores 16 columns of its TMEM lane.
+          tc_fence_after();
+          const int q = warp & 3;
+          const int hs = (warp - kConvWarp0) >> 2;
+          const uint8_t* src = wp + (2 * hs) * 2048 + (q * 32 + lane) * 16;
+          uint4 w[2];
+#pragma unroll
+          for (int j = 0; j < 2; ++j) w[j] = *reinterpret_cast<const uint4*>(src + j * 2048);
+          uint32_t v[16];
+#pragma unroll
+          for (int j = 0; j < 2; ++j) {
+            v[8 * j + 0] = widen_lo(w[j].x);
+            v[8 * j + 1] = widen_hi(w[j].x);
+            v[8 * j + 2] = widen_lo(w[j].y);
+            v[8 * j + 3] = widen_hi(w[j].y);
+            v[8 * j + 4] = widen_lo(w[j].z);
+            v[8 * j + 5] = widen_hi(w[j].z);
+            v[8 * j + 6] = widen_lo(w[j].w);
+            v[8 * j + 7] = widen_hi(w[j].w);
+          }
+          tmem_st16(tmem_base + ((uint32_t)(q * 32) << 16) + a.a_col0 + (uint32_t)(c * 32 + hs * 16), v);
+          tmem_st_wait();
+          tc_fence_before();
+        } else if constexpr (kATmem) {
           // Warp (lane quarter q, half hs) widens k-block hs of rows 32q..32q+31: each
           // thread reads its row's 64 packed bytes (4 chunks of 32 k) and stores 32 columns
           // of its TMEM lane.
@@ -499,12 +545,20 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
           // = 32 weights) into swizzled chunks 2jj and 2jj + 1 of row r.  All loads are
           // issued before any store.
           uint4 w[2 * KPS];
+          if (ctid == 0 && gc == 8) DPTQ_TRACE_CLOCK(tr, 230);
 #pragma unroll
           for (int i = 0; i < 2 * KPS; ++i) {
             const int p = i * kConvThreads + ctid;   // 16-byte unit: tile p >> 9
             const int qq = p & 511;
             w[i] = *reinterpret_cast<const uint4*>(wp + (p >> 9) * kWTileBytes + (qq & 3) * 2048 + (qq >> 2) * 16);
           }
+#ifdef DPTQ_TRACE
+          if (ctid == 0 && gc == 8) {
+            volatile uint32_t sink = w[0].x ^ w[2 * KPS - 1].w;
+            (void)sink;
+            DPTQ_TRACE_CLOCK(tr, 231);
+          }
+#endif
 #pragma unroll
           for (int i = 0; i < 2 * KPS; ++i) {
             const int p = i * kConvThreads + ctid;
@@ -516,10 +570,13 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
             *reinterpret_cast<uint4*>(row + (((j0 + 1) ^ (r & 7)) << 4)) =
                 make_uint4(widen_lo(w[i].z), widen_hi(w[i].z), widen_lo(w[i].w), widen_hi(w[i].w));
           }
+          if (ctid == 0 && gc == 8) DPTQ_TRACE_CLOCK(tr, 232);
           fence_proxy_async_smem();
+          if (ctid == 0 && gc == 8) DPTQ_TRACE_CLOCK(tr, 233);
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(&cfull[c]);
+        if (ctid == 0 && gc == 8) DPTQ_TRACE_CLOCK(tr, 234);
         if (ctid == 0 && gc < 16) DPTQ_TRACE_POINT(tr, 56 + gc);
       }
       if (!ok) break;
@@ -592,17 +649,23 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
       // lane stores 4 consecutive channels of one token (8 bytes instead of four 2-byte
       // stores).  Token scales come from shared memory for tiles of up to 64 tokens, else
       // from the (cached) global array.
-      auto write_out = [&](int c0, const int (&v)[16]) {
+      // vf[i] = fp32(acc) of token c0 + i (the caller's exact conversion); v, if given,
+      // the int32 accumulators for the optional dump.
+      auto write_out = [&](int c0, const float (&vf)[16], const int* v) {
         __half hv[16];
 #pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          const float sav = NT <= 64 ? sa_sh[c0 + i] : __shfl_sync(0xffffffffu, sa_grp, (c0 & 31) + i);
-          hv[i] = __float2half_rn(__fmul_rn(__fmul_rn(__int2float_rn(v[i]), sav), swn));
+        for (int i = 0; i < 16; i += 2) {
+          const float sa0 = NT <= 64 ? sa_sh[c0 + i] : __shfl_sync(0xffffffffu, sa_grp, (c0 & 31) + i);
+          const float sa1 = NT <= 64 ? sa_sh[c0 + i + 1] : __shfl_sync(0xffffffffu, sa_grp, (c0 & 31) + i + 1);
+          const __half2 h2 = __floats2half2_rn(__fmul_rn(__fmul_rn(vf[i], sa0), swn),
+                                               __fmul_rn(__fmul_rn(vf[i + 1], sa1), swn));
+          hv[i] = __low2half(h2);
+          hv[i + 1] = __high2half(h2);
         }
         if (acc_g != nullptr && n < a.N) {
 #pragma unroll
           for (int i = 0; i < 16; ++i)
-            if (m0 + c0 + i < a.M) acc_g[(size_t)(m0 + c0 + i) * a.N + n] = v[i];
+            if (m0 + c0 + i < a.M) acc_g[(size_t)(m0 + c0 + i) * a.N + n] = v != nullptr ? v[i] : __float2int_rn(vf[i]);
         }
         if (a.out_vec) {
           __half* xw = xpose + q * 128;
@@ -663,10 +726,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
           }
           if (etid == 0) DPTQ_TRACE_POINT(tr, c == 0 ? 4 : 119);
           if (finish) {
-            int acc[16];
+            // f * 2^9 is the exact integer accumulator (below 2^24 in one segment), so it
+            // is already fp32(acc).
+            float vf[16];
 #pragma unroll
-            for (int i = 0; i < 16; ++i) acc[i] = __float2int_rn(f[i] * 512.f);
-            write_out(c, acc);
+            for (int i = 0; i < 16; ++i) vf[i] = f[i] * 512.f;
+            write_out(c, vf, nullptr);
           } else {
 #pragma unroll
             for (int j = 0; j < 4; ++j)
@@ -711,7 +776,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
             for (int i = 0; i < 16; ++i) acc[i] += __float2int_rn(__uint_as_float(r[i]) * 512.f);
           }
           if (finish) {
-            write_out(c0, acc);
+            float vf[16];
+#pragma unroll
+            for (int i = 0; i < 16; ++i) vf[i] = __int2float_rn(acc[i]);
+            write_out(c0, vf, acc);
           } else {
 #pragma unroll
             for (int i = 0; i < 16; ++i) atomicAdd(wsl + (c0 + i) * 128 + q * 32 + lane, acc[i]);
@@ -741,27 +809,31 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
         if (flag[1]) {
 #pragma unroll 1
           for (int c0 = 0; c0 < NT; c0 += 16) {
-            int v[16];
             if (NT > 64 && (c0 & 31) == 0) sa_grp = sa_group(c0);
+            float vf[16];
             if (f32) {
 #pragma unroll
               for (int j = 0; j < 4; ++j) {
                 const float4 t = __ldcg(reinterpret_cast<const float4*>(wslf + (c0 / 4 + j) * 512));
-                v[4 * j] = __float2int_rn(t.x * 512.f);
-                v[4 * j + 1] = __float2int_rn(t.y * 512.f);
-                v[4 * j + 2] = __float2int_rn(t.z * 512.f);
-                v[4 * j + 3] = __float2int_rn(t.w * 512.f);
+                vf[4 * j] = t.x * 512.f;   // exact: one segment's sums are below 2^24 units
+                vf[4 * j + 1] = t.y * 512.f;
+                vf[4 * j + 2] = t.z * 512.f;
+                vf[4 * j + 3] = t.w * 512.f;
               }
 #pragma unroll
               for (int j = 0; j < 4; ++j)
                 __stcg(reinterpret_cast<float4*>(wslf + (c0 / 4 + j) * 512), make_float4(0.f, 0.f, 0.f, 0.f));
+              write_out(c0, vf, nullptr);
             } else {
+              int v[16];
 #pragma unroll
               for (int i = 0; i < 16; ++i) v[i] = __ldcg(wsl + (c0 + i) * 128 + q * 32 + lane);
 #pragma unroll
               for (int i = 0; i < 16; ++i) __stcg(wsl + (c0 + i) * 128 + q * 32 + lane, 0);
+#pragma unroll
+              for (int i = 0; i < 16; ++i) vf[i] = __int2float_rn(v[i]);
+              write_out(c0, vf, v);
             }
-            write_out(c0, v);
           }
         }
         if (etid == 0) {
@@ -802,7 +874,7 @@ int gemm_pick_nt(int M, int bits, int KB) {
   if (M <= 32) return 32;
   if (M <= 64) return 64;
   if (M <= 128 || bits == 8) return 128;
-  return 256;
+  return 192;
 }
 
 // Token tiles of up to 64 columns stream weights (decode): two k-blocks per stage to
@@ -833,18 +905,18 @@ bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan, i
   int seg_iters, segs;
   seg_plan(kps, seg_iters, segs);
   while (nt > 16 && nt * segs > 512) {
-    nt >>= 1;
+    nt = nt == 192 ? 128 : nt >> 1;
     if (kps_for(nt) != kps && KB % kps_for(nt) == 0) {
       kps = kps_for(nt);
       seg_plan(kps, seg_iters, segs);
     }
   }
   if (nt * segs > 512) return false;
-  // Widened weights live in TMEM for two-block stages (A operand read from TMEM; 4 slots
-  // of 64 columns after the accumulators), else in shared memory: as many slots as fit
-  // next to at least 4 bulk-copy stages (the converters may run that far ahead of MMA
-  // completion).
-  const bool a_tmem = kps == 2;
+  // Widened weights live in TMEM for two-block stages and 192-token tiles (A operand
+  // read from TMEM; 4 slots of 32 columns per k-block after the accumulators), else in
+  // shared memory: as many slots as fit next to at least 4 bulk-copy stages (the
+  // converters may run that far ahead of MMA completion).
+  const bool a_tmem = a_in_tmem(nt, kps);
   int conv_slots = kMaxConvSlots;
   if (!a_tmem)
     while (conv_slots > 2 && smem_for(nt, kps, 4, planes, conv_slots) > kSmemLimit) --conv_slots;
@@ -952,6 +1024,7 @@ cudaError_t launch_gemm(const GemmPlan& plan, cudaStream_t s, bool pdl) {
     case 32: return launch_nt<32, 1>(plan, s, pdl);
     case 64: return launch_nt<64, 1>(plan, s, pdl);
     case 128: return launch_nt<128, 1>(plan, s, pdl);
+    case 192: return launch_nt<192, 1>(plan, s, pdl);
     case 256: return launch_nt<256, 1>(plan, s, pdl);
     default: return cudaErrorInvalidValue;
   }
