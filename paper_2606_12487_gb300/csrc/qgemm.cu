@@ -878,9 +878,11 @@ int gemm_pick_nt(int M, int bits, int KB) {
 }
 
 // Token tiles of up to 64 columns stream weights (decode): two k-blocks per stage to
-// halve the per-byte barrier and conversion overhead.  Wider tiles are MMA-bound and
-// keep one k-block per stage for a deeper ring.
-static int kps_for(int nt) { return nt <= 64 ? 2 : 1; }
+// halve the per-byte barrier and conversion overhead.  192-token tiles (weights in
+// tensor memory) take two as well: their MMA warp would otherwise spend more time per
+// k-block on barrier waits and commits than the tensor pipe spends on the MMAs.  Other
+// wide tiles keep one k-block per stage for a deeper ring.
+static int kps_for(int nt) { return nt <= 64 || nt == 192 ? 2 : 1; }
 
 static int smem_for(int nt, int kps, int stages, int planes, int conv_slots) {
   return 1024 + conv_slots * kps * kConvBytes + stages * kps * (planes * nt * 128 + kWTileBytes) + kBarrierBytes;
@@ -920,6 +922,8 @@ bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan, i
   int conv_slots = kMaxConvSlots;
   if (!a_tmem)
     while (conv_slots > 2 && smem_for(nt, kps, 4, planes, conv_slots) > kSmemLimit) --conv_slots;
+  else   // room for two accumulators next to the slots
+    while (conv_slots > 2 && 2 * nt * segs + conv_slots * kps * 32 > 512) --conv_slots;
   const int smem_conv = a_tmem ? 0 : conv_slots;
   // A fused launch needs two-block stages (weights widened into TMEM) and room for one
   // row's rotation scratch next to at least 3 stages.
@@ -1016,6 +1020,7 @@ cudaError_t launch_gemm(const GemmPlan& plan, cudaStream_t s, bool pdl) {
       case 16: return launch_nt<16, 2>(plan, s, pdl);
       case 32: return launch_nt<32, 2>(plan, s, pdl);
       case 64: return launch_nt<64, 2>(plan, s, pdl);
+      case 192: return launch_nt<192, 2>(plan, s, pdl);
       default: return cudaErrorInvalidValue;
     }
   }
