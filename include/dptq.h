@@ -201,6 +201,25 @@ dptq_status dptq_qgemm_codes(dptq_handle h, const void* codes, const float* scal
  * inputs / max_N outputs, so that later calls allocate nothing.  Synchronous. */
 dptq_status dptq_reserve(int max_M, int max_K, int max_N);
 
+/* The GEMM launch plan the library would use for M tokens, N outputs, K inputs at
+ * `bits` activation bits on a GPU with num_sms SMs (host only: no GPU is needed or
+ * touched).  fused != 0 plans the one-launch decode kernel that rotates and quantizes
+ * the token rows itself (dptq_qlinear additionally uses it only for K <= 16384 and
+ * when its token padding equals the two-launch plan's).  Writes DPTQ_PLAN_INFO_LEN
+ * ints to info (host memory, caller-owned), in this order:
+ *   0 token tile NT (MMA N)         1 k-blocks of 128 per stage     2 padded tokens M_pad
+ *   3 grid (CTAs)                   4 dynamic shared memory bytes   5 bulk-copy stages
+ *   6 widened-weight slots          7 widened weights in TMEM (1) or shared memory (0)
+ *   8 TMEM accumulator buffers      9 exact-accumulation segments   10 stages per segment
+ *   11 TMEM columns allocated       12 first TMEM column of the weight slots (= the
+ *   accumulators' columns)          13 stages per tile (KI)         14 weight tiles (N/128)
+ *   15 token tiles                  16 tiles processed whole        17 stream-K stages
+ *   (saturated at INT_MAX)          18 parts per token row (fused)  19 fused (1/0).
+ * INVALID_ARG for sizes < 1, bits not 4/8, a null or short info; UNSUPPORTED when no
+ * plan fits (e.g. a fused plan for more than 64 tokens). */
+#define DPTQ_PLAN_INFO_LEN 20
+dptq_status dptq_plan_info(int M, int N, int K, int bits, int num_sms, int fused, int* info, int info_len);
+
 /* Copy the packed weights out in the public layout: wq_host uint8 [N][K/2] (same
  * nibble format as 4-bit activation codes) and sw_host float [N].  Either may be
  * NULL.  Synchronous (test access). */

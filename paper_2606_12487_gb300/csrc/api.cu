@@ -506,6 +506,23 @@ dptq_status dptq_sensitivity_policy(const float* x, const float* dx, int L, int 
   return DPTQ_OK;
 }
 
+dptq_status dptq_plan_info(int M, int N, int K, int bits, int num_sms, int fused, int* info, int info_len) {
+  if (M < 1 || N < 1 || K < 1 || num_sms < 1) return fail(DPTQ_ERR_INVALID_ARG, "sizes must be >= 1");
+  if (bits != 4 && bits != 8) return fail(DPTQ_ERR_INVALID_ARG, "bits must be 4 or 8");
+  if (info == nullptr || info_len < DPTQ_PLAN_INFO_LEN) return fail(DPTQ_ERR_INVALID_ARG, "info too short");
+  GemmPlan plan{};
+  if (!plan_gemm(M, N, round_up(K, kKBlock), bits, num_sms, plan, fused ? kRQPartSmemBytes : 0))
+    return fail(DPTQ_ERR_UNSUPPORTED, "no GEMM plan for this shape");
+  const GemmArgs& g = plan.args;
+  const long long sk = g.sk_iters;
+  const int v[DPTQ_PLAN_INFO_LEN] = {plan.nt, plan.kps, plan.M_pad, plan.grid, plan.smem_bytes, g.stages,
+                                     g.conv_slots, plan.a_tmem ? 1 : 0, g.nbuf, g.segs, g.seg_iters,
+                                     (int)g.tmem_cols, (int)g.a_col0, g.KI, g.n_wtiles, g.m_tiles, g.dp_tiles,
+                                     sk > 0x7fffffffLL ? 0x7fffffff : (int)sk, g.rq_np, plan.fused ? 1 : 0};
+  for (int i = 0; i < DPTQ_PLAN_INFO_LEN; ++i) info[i] = v[i];
+  return DPTQ_OK;
+}
+
 dptq_status dptq_reserve(int max_M, int max_K, int max_N) {
   if (max_M < 0 || max_K < 0 || max_N < 0) return fail(DPTQ_ERR_INVALID_ARG, "sizes must be >= 0");
   int dev;

@@ -130,7 +130,8 @@ struct GemmArgs {
 
 struct GemmPlan {
   bool fused;     // rotation + quantization inside the GEMM launch
-  int nt;          // token tile (MMA N): 16, 32, 64, 128 or 256
+  bool a_tmem;    // widened weights (MMA A operand) in tensor memory, else shared memory
+  int nt;          // token tile (MMA N): 16, 32, 64, 128, 192 or 256
   int kps;         // k-blocks of 128 per pipeline stage (1 or 2)
   int M_pad;
   int grid;

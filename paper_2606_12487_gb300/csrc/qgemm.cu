@@ -952,6 +952,7 @@ bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan, i
   if (tiles >= 2LL * G) dp = (tiles / G - 1) * G;
 
   plan.fused = fused;
+  plan.a_tmem = a_tmem;
   plan.nt = nt;
   plan.kps = kps;
   plan.M_pad = M_pad;

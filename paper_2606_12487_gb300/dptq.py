@@ -25,7 +25,7 @@ EXPORTS = ("dptq_pack_weights", "dptq_rotate_quant_act", "dptq_rotate_act", "dpt
            "dptq_qgemm_codes", "dptq_reserve", "dptq_get_packed", "dptq_get_shape",
            "dptq_last_device_error", "dptq_destroy", "dptq_status_str", "dptq_last_error_message",
            "dptq_pack_weights_rh", "dptq_rotate_quant_act_rh", "dptq_rotate_act_rh", "dptq_kv4_quantize",
-           "dptq_sensitivity_policy")
+           "dptq_sensitivity_policy", "dptq_plan_info")
 
 
 class DptqError(RuntimeError):
@@ -70,6 +70,7 @@ def load(build_if_missing: bool = True):
                 "dptq_kv4_quantize": ([P, I, I, I, P, P, P], I),
                 "dptq_sensitivity_policy": ([P, P, I, I, I, I, ctypes.c_double, ctypes.c_double, ctypes.c_double,
                                              P, P, P, P], I),
+                "dptq_plan_info": ([I, I, I, I, I, I, ctypes.POINTER(I), I], I),
             }
             for name, (args, res) in sig.items():
                 fn = getattr(lib, name)
@@ -274,6 +275,18 @@ def dptq_qgemm_codes(layer: QLinear, codes, scales, bits: int, out, acc=None, st
 
 def dptq_reserve(max_M: int, max_K: int, max_N: int = 0):
     _check(load().dptq_reserve(max_M, max_K, max_N))
+
+
+PLAN_INFO_FIELDS = ("nt", "kps", "M_pad", "grid", "smem_bytes", "stages", "conv_slots", "a_tmem", "nbuf",
+                    "segs", "seg_iters", "tmem_cols", "acc_cols", "KI", "n_wtiles", "m_tiles", "dp_tiles",
+                    "sk_iters", "rq_np", "fused")
+
+
+def dptq_plan_info(M: int, N: int, K: int, bits: int, num_sms: int, fused: bool = False) -> dict:
+    """The GEMM launch plan for a shape (host only, no GPU): a dict of PLAN_INFO_FIELDS."""
+    buf = (ctypes.c_int * len(PLAN_INFO_FIELDS))()
+    _check(load().dptq_plan_info(M, N, K, bits, num_sms, 1 if fused else 0, buf, len(PLAN_INFO_FIELDS)))
+    return dict(zip(PLAN_INFO_FIELDS, list(buf)))
 
 
 def dptq_get_packed(layer: QLinear):
