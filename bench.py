@@ -424,8 +424,12 @@ def run_shapes(args):
         gemm_b = wbytes + 4 * N + M * K * bits // 8 + 4 * M + 2 * M * N
         ql_b = wbytes + 4 * N + 2 * M * K + 2 * M * N
         ops = 2 * M * N * K
+        # rotate + quantize: the fp16 row in, b-bit codes and a scale out (algorithmic bytes;
+        # the GEMM operand planes it actually writes hold one byte per code and plane)
+        q_b = 2 * M * K + M * K * bits // 8 + 4 * M
         r = {"shape": label, "M": M, "N": N, "K": K, "had_block": B, "bits": bits, "weight_copies": copies,
-             "quantize_us": t_q, "gemm_us": t_g, "qlinear_us": t_l,
+             "quantize_us": t_q, "gemm_us": t_g, "qlinear_us": t_l, "quantize_gbs": q_b / t_q / 1e3,
+             "quantize_hbm_frac": q_b / t_q / 1e3 / hbm,
              "gemm_gbs": gemm_b / t_g / 1e3, "qlinear_gbs": ql_b / t_l / 1e3,
              "gemm_tops": ops / t_g / 1e6, "qlinear_tops": ops / t_l / 1e6}
         if M <= 64:
@@ -512,13 +516,63 @@ def stack_time_from(wl, times):
     return sum(times[(gi, wl.bits(li))] for li in range(wl.layers) for gi in range(n_groups))
 
 
-def cpu_baseline(wl, budget_s=12.0):
+def cpu_baseline(wl, budget_s=12.0, all_cores_budget_s=6.0):
     times, calls = oracle_sample_times(wl, budget_s)
     t_stack = stack_time_from(wl, times)
-    return {"value": 1.0 / t_stack, "unit": UNIT, "cores": 1, "kind": "oracle",
+    line = {"value": 1.0 / t_stack, "unit": UNIT, "cores": 1, "kind": "oracle",
             "sample": f"1 token through each of the 4 projection groups at 4 and 8 bits ({calls} oracle calls, "
                       f"~{budget_s:.0f} s), weights as random int4 codes; 32-layer stack time summed from the "
-                      "per-group medians with the layer mask"}
+                      "per-group medians with the layer mask",
+            "host": host_cpu()}
+    try:
+        line["all_cores"] = cpu_baseline_all_cores(wl, all_cores_budget_s)
+    except Exception as e:   # the single-core figure stands on its own
+        line["all_cores"] = {"unavailable": f"{type(e).__name__}: {e}"}
+    return line
+
+
+def host_cpu():
+    """Core count and CPU model of this host (the model line of /proc/cpuinfo where present)."""
+    import platform
+    model = None
+    try:
+        with open("/proc/cpuinfo") as f:
+            for ln in f:
+                key = ln.split(":", 1)[0].strip().lower()
+                if key in ("model name", "cpu model", "hardware") and ":" in ln:
+                    model = ln.split(":", 1)[1].strip()
+                    break
+    except OSError:
+        pass
+    return {"nproc": usable_cores(), "machine": platform.machine(), "cpu_model": model or platform.processor() or None}
+
+
+def usable_cores():
+    """Cores this process may run on (its affinity set; the machine's count as a fallback)."""
+    try:
+        return len(os.sched_getaffinity(0))
+    except (AttributeError, OSError):
+        return os.cpu_count() or 1
+
+
+def _oracle_worker(budget_s):
+    """One process of the all-cores oracle timing: the single-core sample, returned as the
+    stack time of one token stream."""
+    wl = _inputs().llama2_7b_decode()
+    times, calls = oracle_sample_times(wl, budget_s)
+    return stack_time_from(wl, times), calls
+
+
+def cpu_baseline_all_cores(wl, budget_s):
+    """The same oracle sample in one process per core at once (spawned, so no CUDA state is
+    inherited): independent token streams, tokens/s summed over the processes."""
+    import multiprocessing as mp
+    n = min(64, usable_cores())
+    with mp.get_context("spawn").Pool(n) as pool:
+        res = pool.map(_oracle_worker, [budget_s] * n)
+    return {"value": sum(1.0 / t for t, _ in res), "unit": UNIT, "cores": n,
+            "sample": f"{n} processes, each the single-core sample for ~{budget_s:.0f} s "
+                      f"({sum(c for _, c in res)} oracle calls in all); one token stream per process"}
 
 
 def run_reference(args):
