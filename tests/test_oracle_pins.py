@@ -332,6 +332,23 @@ def test_historical_snr_exact_grid(orc):
     assert abs(snr - 10 * math.log10(14.0 / 1e-6)) < 1e-9
 
 
+def test_historical_snr_and_jump_ratio_two_token_closed_form(orc):
+    # Token A: x + dx = [7, 3.5, 0, 0], so s = 1 at 4 bits and the tie 3.5 rounds to 4;
+    # xhat - x = Q(x + dx) - (x + dx) = [0, 0.5, 0, 0]: the numerator is |x|^2 = 30 (not
+    # |xhat|^2 = 32.25), the error 0.25.  Token B: x + dx = [7, 0, 0, 0] is on the grid.
+    # The layer value is the mean of the per-token values in dB (Eq. 11), and JR the mean
+    # of the per-token ratios (Eq. 9).
+    eps = 1e-6
+    x = np.array([[1.0, 2.0, 3.0, 4.0], [2.0, 0.0, 0.0, 0.0]], dtype=np.float32)
+    dx = np.array([[6.0, 1.5, -3.0, -4.0], [5.0, 0.0, 0.0, 0.0]], dtype=np.float32)
+    jr, snr = orc.residual_stats(x, dx, 4, eps=eps)
+    snr_a = 10 * math.log10(30.0 / (0.25 + eps))
+    snr_b = 10 * math.log10(4.0 / eps)
+    assert abs(snr - (snr_a + snr_b) / 2) < 1e-9
+    jr_ref = (math.sqrt(63.25) / (math.sqrt(30.0) + eps) + 5.0 / (2.0 + eps)) / 2
+    assert abs(jr - jr_ref) < 1e-12
+
+
 def test_sensitive_set_golden():
     # Eq. 21 instantiated for the layer counts of the workloads (0-indexed masks)
     gold = {int(a): [int(v) for v in b.split()] for a, b in
