@@ -111,7 +111,9 @@ def run_codes_gemm(dp, orc, layer, codes, sa, bits):
 # rotation of the weights cheap.
 GEMM_CASES = [(16, 512, 256, 32), (1, 4096, 4096, 64), (8, 1024, 4096, 64), (33, 1024, 4096, 64),
               (130, 256, 1024, 32), (300, 384, 512, 32), (64, 128, 11008, 256), (17, 48, 160, 32),
-              (2048, 5120, 256, 32)]
+              (2048, 5120, 256, 32),
+              # 192-token tiles with an odd number of k-blocks: one k-block per stage
+              (200, 256, 384, 128)]
 
 
 @pytest.mark.parametrize("bits", [4, 8])
