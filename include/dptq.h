@@ -38,8 +38,11 @@
  *     {4, 8}.  Violations return
  *     DPTQ_ERR_INVALID_ARG (bits, null pointers, negative sizes) or
  *     DPTQ_ERR_UNSUPPORTED (shape).  M == 0 is a no-op.
- *   - No exception crosses this boundary.  CUDA errors map to DPTQ_ERR_CUDA; the
- *     message of the last failure on the calling thread is dptq_last_error_message().
+ *   - No exception crosses this boundary.  CUDA errors map to DPTQ_ERR_CUDA (failed
+ *     device allocations to DPTQ_ERR_OOM); the message of the last failure on the calling
+ *     thread is dptq_last_error_message().  For tests of the out-of-memory path, the
+ *     environment variable DPTQ_FAULT_ALLOC=n makes the n-th device allocation the
+ *     library attempts in the process fail as out of memory (no cudaMalloc is made).
  *   - Device-side waits are bounded: a pipeline wait that exceeds about one second
  *     makes the kernel record an error word and return; dptq_last_device_error()
  *     reports it as DPTQ_ERR_TIMEOUT.
@@ -155,7 +158,11 @@ dptq_status dptq_sensitivity_policy(const float* x, const float* dx, int L, int 
  * x_fp16: device [M][K]; out_fp16: device [M][N] (written; any alignment, a 16-byte
  * aligned pointer is written 8 bytes at a time).  Asynchronous.
  * Uses the library's per-device scratch (grown on demand; call dptq_reserve before
- * capturing into a CUDA graph so that no allocation happens during capture).
+ * capturing into a CUDA graph so that no allocation happens during capture).  Growth
+ * never frees memory: a call that needs more scratch than the device holds allocates new,
+ * at least twice larger buffers and keeps the superseded ones allocated until the process
+ * exits, so work enqueued earlier and graphs captured earlier (which keep the old
+ * addresses) stay valid.
  * For token tiles of up to 64 rows (M <= 64) whose rotation fits next to the GEMM's
  * pipeline in one CTA's shared memory, rotation, quantization and GEMM run as ONE
  * kernel launch (the environment variable DPTQ_FUSED=0 selects the two-launch
@@ -183,11 +190,14 @@ dptq_status dptq_qlinear_gemm(dptq_handle h, int M, int bits, void* out_fp16, vo
  * an allocating library routine.
  * Limits: M <= 32 tokens and K <= 16384; larger shapes return DPTQ_ERR_UNSUPPORTED.
  * The first call on a device looks the array up (cudaGetSymbolAddress) and zeroes it,
- * synchronously; make that first call before any stream capture.
+ * synchronously; make that first call before any stream capture.  That first call is
+ * also when the CUDA driver brings the array's device memory in (modules load lazily),
+ * so make it, or a warm-up call, before the caller's own pool takes the device memory.
  * All calls share the array: calls whose kernels overlap on the GPU (for example on
  * two streams without ordering between them) race and corrupt each other's results.
- * A bounded-wait timeout inside this call is recorded in the array, not in the word
- * that dptq_last_device_error reads. */
+ * A bounded-wait timeout inside this call is recorded in the array's own error word;
+ * dptq_last_device_error reports it (TIMEOUT) and clears the array's error word, split-tile
+ * sums and counters, without allocating. */
 dptq_status dptq_qlinear_static(dptq_handle h, const void* x_fp16, int M, int bits, void* out_fp16,
                                 void* stream);
 
@@ -229,8 +239,19 @@ dptq_status dptq_get_packed(dptq_handle h, void* wq_host, float* sw_host);
 dptq_status dptq_get_shape(dptq_handle h, int* N, int* K, int* had_block);
 
 /* Synchronize the device and report (and clear) the device error word set by a
- * bounded wait that gave up: DPTQ_OK or DPTQ_ERR_TIMEOUT.  `h` may be NULL. */
+ * bounded wait that gave up: DPTQ_OK or DPTQ_ERR_TIMEOUT.  `h` may be NULL.  Covers the
+ * per-device scratch of the allocating calls and the fixed array of dptq_qlinear_static;
+ * after a timeout it also zeroes the split-tile sums and counters the aborted kernel may
+ * have left, so that later calls start clean. */
 dptq_status dptq_last_device_error(dptq_handle h);
+
+/* Test hook: the activation-plane and scale buffers of the current device's scratch,
+ * current ones first, then the ones that growth superseded (newest first).  Writes up to
+ * `max` entries: ptrs[i] (device address), bytes[i], and allocated[i] = 1 when the CUDA
+ * runtime still reports ptrs[i] as a device allocation; *count = the number of buffers
+ * held.  Host memory, caller-owned.  INVALID_ARG for a null count, or null arrays with
+ * max > 0. */
+dptq_status dptq_scratch_buffers(void** ptrs, size_t* bytes, int* allocated, int max, int* count);
 
 /* Release a handle and its device memory.  NULL is ignored.  Must not be called
  * while work using the handle is still running. */

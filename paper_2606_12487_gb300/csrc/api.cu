@@ -93,6 +93,10 @@ RQArgs make_rq(const void* x, int rows_in, int rows_out, int K, int KB, int B, i
 
 // Per-device scratch shared by the online calls: E4M3 activation planes, per-token
 // scales, split-tile partial sums and their counters, and the device error word.
+// Activation planes and scales grow on demand.  A buffer that growth supersedes is never
+// freed: work enqueued earlier, or captured into a CUDA graph, may still read or write
+// it, so it stays allocated (in `retired`) until the process exits.  Growth is geometric
+// (at least doubling), so the retired buffers together hold less than the live ones.
 struct Scratch {
   uint8_t* act = nullptr;
   size_t act_bytes = 0;
@@ -103,6 +107,7 @@ struct Scratch {
   uint32_t* gsync = nullptr;
   int* err = nullptr;
   int num_sms = 0;
+  std::vector<std::pair<void*, size_t>> retired;   // superseded act / sa buffers, still allocated
 };
 std::mutex g_mu;
 std::map<int, Scratch> g_scratch;
@@ -118,6 +123,23 @@ constexpr int kMaxNT = 256;
 // butterflies twice when the row has more than one chunk).
 constexpr int kFusedMaxKPad = 16384;
 
+// Every device allocation of the library goes through here.  Host-side fault injection
+// for tests of the out-of-memory path: with DPTQ_FAULT_ALLOC=n (n >= 1) in the
+// environment, the n-th allocation the library attempts in this process fails as
+// cudaErrorMemoryAllocation without calling cudaMalloc.
+cudaError_t dev_malloc(void** p, size_t bytes) {
+  static const long long fail_at = [] {
+    const char* v = std::getenv("DPTQ_FAULT_ALLOC");
+    return v ? std::atoll(v) : 0LL;
+  }();
+  static long long n = 0;
+  if (fail_at > 0 && ++n == fail_at) {
+    *p = nullptr;
+    return cudaErrorMemoryAllocation;
+  }
+  return cudaMalloc(p, bytes);
+}
+
 // Make sure the device's scratch holds `act_bytes` of activation planes and `sa_count`
 // scales.  Growth allocates, so it is refused while `s` is being captured.
 dptq_status ensure_scratch(int dev, size_t act_bytes, size_t sa_count, cudaStream_t s, Scratch** out) {
@@ -129,30 +151,45 @@ dptq_status ensure_scratch(int dev, size_t act_bytes, size_t sa_count, cudaStrea
   if ((grow_act || grow_sa || first) && capturing(s))
     return fail(DPTQ_ERR_UNSUPPORTED, "scratch must grow during stream capture: call dptq_reserve first");
   if (first) {
-    DPTQ_CUDA(cudaDeviceGetAttribute(&sc.num_sms, cudaDevAttrMultiProcessorCount, dev), "cudaDeviceGetAttribute");
-    const size_t ws_bytes = (size_t)sc.num_sms * kMaxNT * 128 * sizeof(int32_t);
-    DPTQ_CUDA(cudaMalloc(&sc.ws, ws_bytes), "cudaMalloc(ws)");
-    DPTQ_CUDA(cudaMalloc(&sc.counters, sizeof(uint32_t) * (sc.num_sms + 2)), "cudaMalloc(counters)");
-    sc.gsync = sc.counters + sc.num_sms;
-    DPTQ_CUDA(cudaMalloc(&sc.err, sizeof(int)), "cudaMalloc(err)");
-    DPTQ_CUDA(cudaMemset(sc.ws, 0, ws_bytes), "cudaMemset(ws)");
-    DPTQ_CUDA(cudaMemset(sc.counters, 0, sizeof(uint32_t) * (sc.num_sms + 2)), "cudaMemset(counters)");
-    DPTQ_CUDA(cudaMemset(sc.err, 0, sizeof(int)), "cudaMemset(err)");
+    int sms = 0;
+    DPTQ_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev), "cudaDeviceGetAttribute");
+    const size_t ws_bytes = (size_t)sms * kMaxNT * 128 * sizeof(int32_t);
+    int32_t* ws = nullptr;
+    uint32_t* counters = nullptr;
+    int* err = nullptr;
+    cudaError_t e = dev_malloc(reinterpret_cast<void**>(&ws), ws_bytes);
+    if (e == cudaSuccess) e = dev_malloc(reinterpret_cast<void**>(&counters), sizeof(uint32_t) * (sms + 2));
+    if (e == cudaSuccess) e = dev_malloc(reinterpret_cast<void**>(&err), sizeof(int));
+    if (e == cudaSuccess) e = cudaMemset(ws, 0, ws_bytes);
+    if (e == cudaSuccess) e = cudaMemset(counters, 0, sizeof(uint32_t) * (sms + 2));
+    if (e == cudaSuccess) e = cudaMemset(err, 0, sizeof(int));
+    if (e != cudaSuccess) {   // nothing has used these yet: release them and stay uninitialized
+      if (ws) cudaFree(ws);
+      if (counters) cudaFree(counters);
+      if (err) cudaFree(err);
+      return cuda_fail(e, "scratch allocation");
+    }
+    sc.num_sms = sms;
+    sc.ws = ws;
+    sc.counters = counters;
+    sc.gsync = counters + sms;
+    sc.err = err;
   }
-  if (grow_act || grow_sa) DPTQ_CUDA(cudaDeviceSynchronize(), "cudaDeviceSynchronize");
   if (grow_act) {
-    if (sc.act) cudaFree(sc.act);
-    sc.act = nullptr;
-    sc.act_bytes = 0;
-    DPTQ_CUDA(cudaMalloc(&sc.act, act_bytes), "cudaMalloc(act)");
-    sc.act_bytes = act_bytes;
+    const size_t bytes = std::max(act_bytes, 2 * sc.act_bytes);
+    void* p = nullptr;
+    DPTQ_CUDA(dev_malloc(&p, bytes), "cudaMalloc(act)");
+    if (sc.act) sc.retired.emplace_back(sc.act, sc.act_bytes);
+    sc.act = static_cast<uint8_t*>(p);
+    sc.act_bytes = bytes;
   }
   if (grow_sa) {
-    if (sc.sa) cudaFree(sc.sa);
-    sc.sa = nullptr;
-    sc.sa_count = 0;
-    DPTQ_CUDA(cudaMalloc(&sc.sa, sizeof(float) * sa_count), "cudaMalloc(sa)");
-    sc.sa_count = sa_count;
+    const size_t count = std::max(sa_count, 2 * sc.sa_count);
+    void* p = nullptr;
+    DPTQ_CUDA(dev_malloc(&p, sizeof(float) * count), "cudaMalloc(sa)");
+    if (sc.sa) sc.retired.emplace_back(sc.sa, sizeof(float) * sc.sa_count);
+    sc.sa = static_cast<float*>(p);
+    sc.sa_count = count;
   }
   *out = &sc;
   return DPTQ_OK;
@@ -210,6 +247,14 @@ bool fused_allowed() {
   return on;
 }
 
+bool l2_prefetch_allowed() {
+  static const bool on = [] {
+    const char* v = std::getenv("DPTQ_L2PF");
+    return !(v && v[0] == '0');
+  }();
+  return on;
+}
+
 // Record the message returned by dptq_last_error_message for this thread.
 void set_error_message(const std::string& m) { g_msg = m; }
 }  // namespace dptq
@@ -261,16 +306,16 @@ dptq_status pack_weights_impl(const void* W_fp16, int N, int K, int had_block, c
   }
   const size_t wt_bytes = (size_t)(h->N_pad / 128) * h->KB * kWTileBytes;
   void* tmp = nullptr;
-  cudaError_t e = cudaMalloc(&h->wt, wt_bytes);
-  if (e == cudaSuccess) e = cudaMalloc(&h->sw, sizeof(float) * h->N_pad);
+  cudaError_t e = dev_malloc(reinterpret_cast<void**>(&h->wt), wt_bytes);
+  if (e == cudaSuccess) e = dev_malloc(reinterpret_cast<void**>(&h->sw), sizeof(float) * h->N_pad);
   if (e == cudaSuccess && signs_host != nullptr) {
-    e = cudaMalloc(&h->signs, (size_t)h->K_pad);
+    e = dev_malloc(reinterpret_cast<void**>(&h->signs), (size_t)h->K_pad);
     if (e == cudaSuccess) e = cudaMemset(h->signs, 1, (size_t)h->K_pad);
     if (e == cudaSuccess) e = cudaMemcpy(h->signs, signs_host, (size_t)K, cudaMemcpyHostToDevice);
   }
   const void* src = W_fp16;
   if (e == cudaSuccess && !w_on_device) {
-    e = cudaMalloc(&tmp, (size_t)N * K * 2);
+    e = dev_malloc(&tmp, (size_t)N * K * 2);
     if (e == cudaSuccess) e = cudaMemcpy(tmp, W_fp16, (size_t)N * K * 2, cudaMemcpyHostToDevice);
     src = tmp;
   }
@@ -584,21 +629,61 @@ dptq_status dptq_last_device_error(dptq_handle h) {
   dptq_status st = current_device(&dev);
   if (st != DPTQ_OK) return st;
   DPTQ_CUDA(cudaDeviceSynchronize(), "cudaDeviceSynchronize");
-  std::lock_guard<std::mutex> lk(g_mu);
-  auto it = g_scratch.find(dev);
-  if (it == g_scratch.end() || it->second.err == nullptr) return DPTQ_OK;
-  Scratch& sc = it->second;
   int word = 0;
-  DPTQ_CUDA(cudaMemcpy(&word, sc.err, sizeof(int), cudaMemcpyDeviceToHost), "cudaMemcpy(err)");
+  {
+    std::lock_guard<std::mutex> lk(g_mu);
+    auto it = g_scratch.find(dev);
+    if (it != g_scratch.end() && it->second.err != nullptr) {
+      Scratch& sc = it->second;
+      DPTQ_CUDA(cudaMemcpy(&word, sc.err, sizeof(int), cudaMemcpyDeviceToHost), "cudaMemcpy(err)");
+      if (word != 0) {
+        // A wait gave up: clear the word, the split-tile sums and every counter (split-tile
+        // arrivals and the fused launch's two grid counters) the aborted kernel may have
+        // left non-zero.
+        DPTQ_CUDA(cudaMemset(sc.err, 0, sizeof(int)), "cudaMemset(err)");
+        DPTQ_CUDA(cudaMemset(sc.ws, 0, (size_t)sc.num_sms * kMaxNT * 128 * sizeof(int32_t)), "cudaMemset(ws)");
+        DPTQ_CUDA(cudaMemset(sc.counters, 0, sizeof(uint32_t) * (sc.num_sms + 2)), "cudaMemset(counters)");
+      }
+    }
+  }
+  // The fixed scratch of dptq_qlinear_static keeps its own error word.
+  int sword = 0;
+  const cudaError_t e = static_scratch_check_reset(dev, &sword);
+  if (e != cudaSuccess) return cuda_fail(e, "static scratch error word");
+  if (word == 0) word = sword;
   if (word == 0) return DPTQ_OK;
-  // A wait gave up: clear the word and the split-tile scratch the aborted kernel may
-  // have left non-zero.
-  DPTQ_CUDA(cudaMemset(sc.err, 0, sizeof(int)), "cudaMemset(err)");
-  DPTQ_CUDA(cudaMemset(sc.ws, 0, (size_t)sc.num_sms * kMaxNT * 128 * sizeof(int32_t)), "cudaMemset(ws)");
-  DPTQ_CUDA(cudaMemset(sc.counters, 0, sizeof(uint32_t) * sc.num_sms), "cudaMemset(counters)");
   char buf[64];
   snprintf(buf, sizeof(buf), "device wait timed out (code 0x%x)", word);
   return fail(DPTQ_ERR_TIMEOUT, buf);
+}
+
+dptq_status dptq_scratch_buffers(void** ptrs, size_t* bytes, int* allocated, int max, int* count) {
+  if (count == nullptr || max < 0 || (max > 0 && (ptrs == nullptr || bytes == nullptr || allocated == nullptr)))
+    return fail(DPTQ_ERR_INVALID_ARG, "null pointer or negative max");
+  int dev;
+  dptq_status st = current_device(&dev);
+  if (st != DPTQ_OK) return st;
+  std::vector<std::pair<void*, size_t>> list;
+  {
+    std::lock_guard<std::mutex> lk(g_mu);
+    auto it = g_scratch.find(dev);
+    if (it != g_scratch.end()) {
+      const Scratch& sc = it->second;
+      if (sc.act) list.emplace_back(sc.act, sc.act_bytes);
+      if (sc.sa) list.emplace_back(sc.sa, sizeof(float) * sc.sa_count);
+      list.insert(list.end(), sc.retired.rbegin(), sc.retired.rend());
+    }
+  }
+  *count = (int)list.size();
+  for (int i = 0; i < (int)list.size() && i < max; ++i) {
+    ptrs[i] = list[i].first;
+    bytes[i] = list[i].second;
+    cudaPointerAttributes at{};
+    const cudaError_t e = cudaPointerGetAttributes(&at, list[i].first);
+    allocated[i] = (e == cudaSuccess && at.type == cudaMemoryTypeDevice) ? 1 : 0;
+    if (e != cudaSuccess) (void)cudaGetLastError();
+  }
+  return DPTQ_OK;
 }
 
 void dptq_destroy(dptq_handle h) {

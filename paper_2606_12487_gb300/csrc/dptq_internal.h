@@ -119,6 +119,7 @@ struct GemmArgs {
   long long sk_iters;  // stream-K iterations (tiles after dp_tiles, times KI)
   uint32_t tmem_cols;
   int out_vec;         // `out` is 16-byte aligned: the epilogue stores 8 channels at a time
+  long long l2_prefetch;  // weight bytes past the first ring stages each CTA requests into L2 up front (0: none)
   // Fused decode launches only: the rotation + quantization of the M_pad token rows
   // (written to `act` / `sa` by the converter warps of CTAs 0, 1, ...) and the two grid
   // counters [rows ready, CTAs done] that order it before the GEMM (zero between launches).
@@ -151,6 +152,14 @@ cudaError_t launch_gemm(const GemmPlan& plan, cudaStream_t s, bool pdl);
 bool pdl_allowed();
 // The fused decode kernel is used unless the environment sets DPTQ_FUSED=0.
 bool fused_allowed();
+// Decode GEMM launches prefetch their weight share into L2 unless DPTQ_L2PF=0.
+bool l2_prefetch_allowed();
+
+// The fixed scratch of dptq_qlinear_static on device `dev`: read its device error word
+// into *word and, when it is non-zero, clear the word, the split-tile sums and the
+// arrival counters (synchronous; no allocation).  *word = 0 when the scratch was never
+// set up on that device.
+cudaError_t static_scratch_check_reset(int dev, int* word);
 
 // Message returned by dptq_last_error_message() on the calling thread.
 void set_error_message(const std::string& m);

@@ -286,6 +286,36 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
       }
       return true;
     };
+    // Decode launches: once the first S stages are requested, the rest of this CTA's
+    // weight share (up to a cap) is requested into L2 in one go, so that HBM streams the
+    // weights while the token rows are rotated and published, instead of only as fast as
+    // the ring frees stages.  Units are visited in processing order; each unit's weight
+    // range is contiguous (tile-major, k-blocks consecutive) and, with one token tile,
+    // belongs to this CTA alone.
+    auto prefetch_share = [&]() {
+      if (a.l2_prefetch <= 0 || !leader) return;
+      UnitIter pit;
+      pit.init(a);
+      Unit pu;
+      long long skip = (long long)S * w_bytes;   // fetched by the ring directly
+      long long budget = a.l2_prefetch;
+      while (budget > 0 && pit.next(pu)) {
+        const int tile_n = pu.tile / a.m_tiles;
+        const uint8_t* base = a.wt + ((size_t)tile_n * a.KB + (size_t)pu.i0 * KPS) * kWTileBytes;
+        long long len = (long long)(pu.i1 - pu.i0) * w_bytes;
+        if (skip >= len) {
+          skip -= len;
+          continue;
+        }
+        base += skip;
+        len -= skip;
+        skip = 0;
+        if (len > budget) len = budget;
+        budget -= len;
+        for (long long off = 0; off < len; off += 32768)
+          bulk_prefetch_l2(base + off, (uint32_t)(len - off < 32768 ? len - off : 32768));
+      }
+    };
     // Weight tiles do not depend on the previous kernel; the first `S` stages are
     // requested before waiting for it and their activation halves are issued once
     // act_ready() returns (also after an abort, so that every armed stage completes).
@@ -319,6 +349,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
           if (g < 16) DPTQ_TRACE_POINT(tr, 24 + g);
         }
         if (!waited && ++npend == S) {
+          prefetch_share();
           if (!act_ready()) ok = false;
           waited = true;
           __syncwarp();
@@ -978,6 +1009,10 @@ bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan, i
   if ((long long)a.sk_iters * G + G >= (1LL << 32) || tiles >= (1LL << 31)) return false;
   a.tmem_cols = cols;
   a.out_vec = 0;
+  // Decode plans (one token tile of at most 64, weights streamed once): each CTA may
+  // request up to 512 KB of its share into L2 ahead of the ring (76 MB over 152 SMs,
+  // within the 129 MB L2).
+  a.l2_prefetch = (nt <= 64 && m_tiles == 1 && l2_prefetch_allowed()) ? 512LL * 1024 : 0;
   a.rq = RQArgs{};
   a.gsync = nullptr;
   // Fused: up to 4 CTAs share each token row (each converts and writes a quarter of it),

@@ -91,6 +91,25 @@ bool pow2(int v) { return v > 0 && (v & (v - 1)) == 0; }
 
 }  // namespace
 
+namespace dptq {
+// A bounded wait that gave up inside dptq_qlinear_static leaves its error word, and
+// possibly split-tile sums and arrival counters, in the fixed array; every later call
+// would start from those.  dptq_last_device_error calls this (after synchronizing the
+// device) to report the word and return the array to its clean state.  No allocation.
+cudaError_t static_scratch_check_reset(int dev, int* word) {
+  *word = 0;
+  if (dev < 0 || dev >= kMaxDevices) return cudaSuccess;
+  std::lock_guard<std::mutex> lk(g_static_mu);
+  const StaticState& st = g_static_state[dev];
+  if (!st.ready) return cudaSuccess;
+  cudaError_t e = cudaMemcpy(word, st.base + kErrOff, sizeof(int), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess || *word == 0) return e;
+  e = cudaMemset(st.base + kWsOff, 0, kWsBytes + kCntBytes + kErrBytes);
+  if (e == cudaSuccess) e = cudaDeviceSynchronize();
+  return e;
+}
+}  // namespace dptq
+
 extern "C" dptq_status dptq_qlinear_static(dptq_handle h, const void* x_fp16, int M, int bits, void* out_fp16,
                                            void* stream) {
   if (!h) return static_fail(DPTQ_ERR_INVALID_ARG, "null handle");

@@ -25,7 +25,7 @@ EXPORTS = ("dptq_pack_weights", "dptq_rotate_quant_act", "dptq_rotate_act", "dpt
            "dptq_qgemm_codes", "dptq_reserve", "dptq_get_packed", "dptq_get_shape",
            "dptq_last_device_error", "dptq_destroy", "dptq_status_str", "dptq_last_error_message",
            "dptq_pack_weights_rh", "dptq_rotate_quant_act_rh", "dptq_rotate_act_rh", "dptq_kv4_quantize",
-           "dptq_sensitivity_policy", "dptq_plan_info")
+           "dptq_sensitivity_policy", "dptq_plan_info", "dptq_scratch_buffers")
 
 
 class DptqError(RuntimeError):
@@ -71,6 +71,8 @@ def load(build_if_missing: bool = True):
                 "dptq_sensitivity_policy": ([P, P, I, I, I, I, ctypes.c_double, ctypes.c_double, ctypes.c_double,
                                              P, P, P, P], I),
                 "dptq_plan_info": ([I, I, I, I, I, I, ctypes.POINTER(I), I], I),
+                "dptq_scratch_buffers": ([ctypes.POINTER(P), ctypes.POINTER(ctypes.c_size_t), ctypes.POINTER(I), I,
+                                          ctypes.POINTER(I)], I),
             }
             for name, (args, res) in sig.items():
                 fn = getattr(lib, name)
@@ -301,3 +303,16 @@ def dptq_get_packed(layer: QLinear):
 
 def dptq_last_device_error():
     _check(load().dptq_last_device_error(None))
+
+
+def dptq_scratch_buffers(max_entries: int = 64):
+    """Test hook: [(device address, bytes, still allocated)] of the current device's
+    activation-plane and scale scratch, current buffers first, then superseded ones."""
+    P = ctypes.c_void_p
+    ptrs = (P * max_entries)()
+    sizes = (ctypes.c_size_t * max_entries)()
+    alloc = (ctypes.c_int * max_entries)()
+    count = ctypes.c_int(0)
+    _check(load().dptq_scratch_buffers(ptrs, sizes, alloc, max_entries, ctypes.byref(count)))
+    n = min(count.value, max_entries)
+    return [(int(ptrs[i] or 0), int(sizes[i]), bool(alloc[i])) for i in range(n)]

@@ -1,0 +1,114 @@
+"""Failure handling of the library on the GPU, without faulting it: allocation failures
+injected on the host (DPTQ_FAULT_ALLOC), scratch growth that must not free memory that
+earlier work still uses, and bounded in-kernel waits that run out."""
+import os
+import subprocess
+import sys
+import textwrap
+
+import pytest
+
+from paper_2606_12487_gb300 import inputs
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def dp():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2606_12487_gb300 import dptq
+    dptq.load()
+    return dptq
+
+
+def test_scratch_growth_keeps_buffers_of_captured_graphs(dp):
+    """A graph captured with the scratch at one size keeps its buffer addresses; a later
+    call that needs more scratch must allocate new buffers and leave the old ones
+    allocated (the host-side query checks that), so replaying the graph stays valid."""
+    wl = inputs.llama2_7b_decode()
+    K, N, B = 2048, 256, 2048
+    layer = dp.dptq_pack_weights(torch.from_numpy(inputs.weights(N, K, layer=2)).cuda(), B)
+    small = torch.from_numpy(inputs.activations(wl, 8, K)).cuda()
+    out_s = torch.empty((8, N), dtype=torch.float16, device="cuda")
+    dp.dptq_qlinear(layer, small, 4, out_s)            # sizes the scratch for this call
+    torch.cuda.synchronize()
+    ref = out_s.clone()
+    s = torch.cuda.Stream()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        dp.dptq_qlinear(layer, small, 4, out_s)
+    before = {p for p, _, alive in dp.dptq_scratch_buffers() if alive}
+    assert before, "no scratch buffers reported"
+    # More tokens than the device's scratch holds (earlier tests in the same process may
+    # have grown it): the scratch must grow.
+    act_bytes = dp.dptq_scratch_buffers()[0][1]
+    M_big = max(40000, act_bytes // (2 * K) + 512)
+    big = torch.from_numpy(inputs.activations(wl, M_big, K)).cuda()
+    out_b = torch.empty((M_big, N), dtype=torch.float16, device="cuda")
+    dp.dptq_qlinear(layer, big, 8, out_b)
+    torch.cuda.synchronize()
+    after = dp.dptq_scratch_buffers()
+    live = {p for p, _, alive in after if alive}
+    assert before <= live, "a buffer captured by the graph was freed by scratch growth"
+    assert len(after) > len(before), "the large call did not grow the scratch"
+    out_s.zero_()
+    g.replay()
+    torch.cuda.synchronize()
+    assert torch.equal(out_s.view(torch.int16), ref.view(torch.int16))
+    dp.dptq_last_device_error()
+    layer.close()
+
+
+def _child(code, fail_at):
+    env = dict(os.environ, DPTQ_FAULT_ALLOC=str(fail_at))
+    r = subprocess.run([sys.executable, "-c", textwrap.dedent(code)], cwd=ROOT, env=env, capture_output=True,
+                       text=True, timeout=600)
+    assert r.returncode == 0, r.stdout + r.stderr
+    return r.stdout
+
+
+CHILD = """
+import torch
+from paper_2606_12487_gb300 import dptq, inputs
+dptq.load()
+W = torch.from_numpy(inputs.weights(256, 1024)).cuda()
+x = torch.from_numpy(inputs.activations(inputs.llama2_7b_decode(), 4, 1024)).cuda()
+out = torch.empty((4, 256), dtype=torch.float16, device="cuda")
+def attempt(fn):
+    try:
+        fn()
+        return "ok"
+    except dptq.DptqError as e:
+        return "oom" if e.status == 4 else f"status{e.status}"
+res = []
+layer = None
+def pack():
+    global layer
+    layer = dptq.dptq_pack_weights(W, 1024)
+res.append(attempt(pack))
+if layer is None:
+    res.append(attempt(pack))
+res.append(attempt(lambda: dptq.dptq_qlinear(layer, x, 4, out)))
+if res[-1] != "ok":
+    res.append(attempt(lambda: dptq.dptq_qlinear(layer, x, 4, out)))
+torch.cuda.synchronize()
+ref = out.clone()
+dptq.dptq_qlinear(layer, x, 4, out)
+torch.cuda.synchronize()
+print(" ".join(res), "same" if torch.equal(out, ref) else "differs")
+"""
+
+
+@pytest.mark.parametrize("fail_at,expect", [(1, "oom ok ok same"), (3, "ok oom ok same"), (5, "ok oom ok same"),
+                                            (6, "ok oom ok same")])
+def test_injected_allocation_failure_reports_oom(fail_at, expect):
+    """The n-th device allocation fails (host-side injection, no real exhaustion): the
+    failing call returns DPTQ_ERR_OOM and leaves nothing half-built, and the same call
+    made again succeeds.  Allocations: 1-2 the handle's packed weights and scales, 3-5
+    the per-device split-tile sums, counters and error word, 6-7 the activation planes
+    and token scales."""
+    out = _child(CHILD, fail_at).strip().splitlines()[-1]
+    assert out == expect, out

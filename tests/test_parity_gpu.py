@@ -54,6 +54,66 @@ def edge_rows(K):
     return inputs.to_f16(rows)
 
 
+# Pairs (a, b): a row with a at position i and b at position j of every Hadamard block
+# rotates to +-(a + b) / sqrt(B) and +-(a - b) / sqrt(B), so y / s = qmax (a - b) / (a + b)
+# wherever H[i][k] != H[j][k].  For (3k, k) that is 3.5 at 4 bits and 63.5 at 8 bits;
+# (27, 1) gives 6.5 at 4 bits: exact rounding ties (Eq. 2, round half to even), half of
+# every row.
+TIE_PAIRS = [(3, 1), (27, 1), (381, 127), (9, 3), (6, 2), (15, 5), (33, 11), (27, 9)]
+
+
+def tie_rows(K, B, n=8):
+    """n fp16 rows whose rotated values sit exactly on half-integers of the code grid."""
+    rows = np.zeros((n, K), dtype=np.float32)
+    for r in range(n):
+        a, b = TIE_PAIRS[r % len(TIE_PAIRS)]
+        i = (7 * r + 3) % B
+        j = (i + 1 + 13 * r) % B
+        for k0 in range(0, K - B + 1, B):
+            rows[r, k0 + i] = a
+            rows[r, k0 + j] = b
+    return inputs.to_f16(rows)
+
+
+def oracle_ties(y_ref, s_ref):
+    """Number of values whose oracle quotient y / s (fp32, as the oracle forms it) is
+    exactly k + 1/2."""
+    s = np.asarray(s_ref, dtype=np.float32)[:, None]
+    ok = s != 0
+    t = np.where(ok, np.asarray(y_ref, dtype=np.float32) / np.where(ok, s, np.float32(1)), np.float32(0))
+    t = np.abs(t.astype(np.float32))
+    return int(np.sum(t - np.floor(t) == 0.5))
+
+
+TIE_CASES = [(256, 256), (4096, 256), (4096, 4096), (2048, 512), (4096, 2048), (11008, 256), (1024, 128)]
+
+
+@pytest.mark.parametrize("bits", [4, 8])
+@pytest.mark.parametrize("K,B", TIE_CASES)
+def test_exact_ties_round_half_even(dp, orc, K, B, bits):
+    """Rows built so that half of their rotated values land exactly on a half-integer of
+    the code grid (Section 2 Eq. 2: the rounding of y / s; Section 4.2 per-token
+    symmetric scale).  The oracle rounds them half to even; the GPU's exact rotation and
+    IEEE-quotient fallback must give the same codes.  For even log2 B the GPU's rotated
+    values are bit-identical to the oracle's, so no mismatch at all is allowed; for odd
+    log2 B the parity contract (tie mismatches off by one, at most 1e-5 of the codes)."""
+    x = tie_rows(K, B)
+    c_ref, s_ref = orc.rotate_quant_act(x, B, bits)
+    y_ref = orc.rotate(x, B)
+    ties = oracle_ties(y_ref, s_ref)
+    assert ties >= x.shape[0] * K // 4, f"only {ties} exact ties in the oracle's quotients"
+    # the oracle's tie codes are the even neighbours
+    t = y_ref.astype(np.float32) / s_ref.astype(np.float32)[:, None]
+    at = np.abs(t) - np.floor(np.abs(t)) == 0.5
+    assert np.all(c_ref[at] % 2 == 0)
+    c, s = gpu_codes(dp, x, B, bits, orc)
+    parity.check_scales(s, s_ref)
+    n = parity.check_codes(c, c_ref, y_ref, s_ref, bits)
+    log2b = B.bit_length() - 1
+    if log2b % 2 == 0:
+        assert n == 0 and np.array_equal(s, s_ref), f"{n} tie mismatches on an even-log2 block"
+
+
 ROT_CASES = [(256, 256, 16), (4096, 4096, 8), (11008, 256, 6), (13824, 1024, 5), (14336, 2048, 4),
              (28672, 4096, 2), (160, 32, 3), (768, 512, 3), (96, 64, 2), (5120, 1024, 4)]
 
@@ -214,6 +274,8 @@ def test_qlinear_ragged_token_counts(dp, orc, M):
     wl = inputs.llama2_7b_decode()
     K, N, B = 1024, 272, 1024
     x = inputs.activations(wl, M, K)
+    if M >= 17:   # exact rounding ties inside a ragged token tile
+        x = np.concatenate([x[:M - 4], tie_rows(K, B, 4)])
     W = inputs.weights(N, K, layer=4, proj=1)
     for bits in (4, 8):
         check_qlinear(dp, orc, x, W, B, bits)
@@ -322,6 +384,16 @@ def test_no_device_error_left(dp):
 
 
 # ----------------------------------------------------------------------------- full-size workloads
+def tile_sample(N, seed):
+    """One output channel from every 128-channel weight tile (a random one per tile), and
+    the first and last channel: every tile's epilogue, and every split-tile reduction of
+    the stream-K work split, is compared with the oracle."""
+    rng = np.random.default_rng(seed)
+    cols = {min(N - 1, t * 128 + int(rng.integers(128))) for t in range((N + 127) // 128)}
+    cols.update({0, N - 1})
+    return np.array(sorted(cols))
+
+
 def sample(n, k, seed, must=()):
     rng = np.random.default_rng(seed)
     pick = set(int(v) for v in rng.choice(n, min(k, n), replace=False))
@@ -337,7 +409,9 @@ def test_llama2_7b_decode_shapes(dp, orc, M, proj):
     p = {pp.name: pp for pp in wl.projs}[proj]
     x = inputs.activations(wl, M, p.K)
     W = inputs.weights(p.N, p.K, layer=0, proj=[pp.name for pp in wl.projs].index(proj))
-    cols = sample(p.N, 48, 5)
+    if M >= 8:   # two rows of exact rounding ties
+        x = np.concatenate([x[:M - 2], tie_rows(p.K, p.had_block, 2)])
+    cols = tile_sample(p.N, 5)
     for bits in (4, 8):
         check_qlinear(dp, orc, x, W, p.had_block, bits, cols=cols)
 
@@ -354,5 +428,43 @@ def test_prefill_and_70b_shapes_sampled(dp, orc, wl_name, proj, M, bits):
     W = inputs.weights(p.N, p.K, layer=1, proj=[pp.name for pp in wl.projs].index(proj))
     hot = [t for t in range(M) if np.abs(x[t].astype(np.float32)).max() > 50]
     rows = sample(M, 24, 7, must=hot[:8])
-    cols = sample(p.N, 24, 8)
+    cols = tile_sample(p.N, 8)
     check_qlinear(dp, orc, x, W, p.had_block, bits, rows=rows, cols=cols)
+
+
+@pytest.mark.parametrize("wl_name,proj,M,bits", [
+    ("llama2-70b", "q", 1, 4), ("llama2-70b", "q", 1, 8), ("llama2-70b", "down", 1, 4),
+    ("llama2-70b", "gate", 64, 4), ("llama3-8b-prefill", "k", 2048, 4), ("llama3-8b-prefill", "v", 2048, 8),
+])
+def test_more_workload_shapes(dp, orc, wl_name, proj, M, bits):
+    """LLaMA-2-70B at one token (the fused decode launch for K = 8192, the two-launch path
+    for the 28672-long down row) and at 64 tokens, and LLaMA-3-8B's GQA k / v projections
+    (N = 1024) in prefill; one channel per weight tile."""
+    wl = inputs.WORKLOADS[wl_name]()
+    p = {pp.name: pp for pp in wl.projs}[proj]
+    x = inputs.activations(wl, M, p.K)
+    W = inputs.weights(p.N, p.K, layer=5, proj=[pp.name for pp in wl.projs].index(proj))
+    hot = [t for t in range(M) if np.abs(x[t].astype(np.float32)).max() > 50]
+    rows = None if M <= 64 else sample(M, 24, 9, must=hot[:8])
+    check_qlinear(dp, orc, x, W, p.had_block, bits, rows=rows, cols=tile_sample(p.N, 10))
+
+
+@pytest.mark.parametrize("wl_name,group,M", [("llama2-7b-decode", "qkv", 32), ("llama2-7b-decode", "gateup", 32),
+                                             ("llama3-8b-prefill", "gateup", 2048)])
+@pytest.mark.parametrize("bits", [4, 8])
+def test_concatenated_group_handles(dp, orc, wl_name, group, M, bits):
+    """The benchmark's concatenated handles: q|k|v (N = 12288) and gate|up (N = 22016) of
+    LLaMA-2-7B at 32 tokens, and LLaMA-3-8B's gate|up (N = 28672) in prefill, packed as one
+    weight matrix (the rows of the group's projections stacked), against the oracle on one
+    channel of every 128-channel tile.  One quantization of x feeds the whole group."""
+    wl = inputs.WORKLOADS[wl_name]()
+    names = [pp.name for pp in wl.projs]
+    projs = [pp for pp in wl.projs if pp.group == group]
+    K, B = projs[0].K, projs[0].had_block
+    W = np.concatenate([inputs.weights(pp.N, pp.K, layer=3, proj=names.index(pp.name)) for pp in projs])
+    x = inputs.activations(wl, M, K)
+    if M <= 64:
+        x = np.concatenate([x[:M - 2], tie_rows(K, B, 2)])
+    hot = [t for t in range(M) if np.abs(x[t].astype(np.float32)).max() > 50]
+    rows = None if M <= 64 else sample(M, 16, 11, must=hot[:4])
+    check_qlinear(dp, orc, x, W, B, bits, rows=rows, cols=tile_sample(W.shape[0], 12))

@@ -1,17 +1,18 @@
 """dptq_qlinear_static, the entry point that allocates no device memory, against
 dptq_qlinear.
 
-Callers whose own memory pool owns the device, or that may not call cudaMalloc once
-they are serving, cannot let the library grow its scratch; dptq_qlinear_static serves
-them from a fixed array inside the library.  This file is collected last, so a failure
-here comes after every other test has run; it also passes on its own in a fresh
-process.
+Some callers cannot let the library allocate device memory when they call it: serving
+runtimes whose own memory pool has already taken the device's memory, and hosts that
+forbid cudaMalloc once they are serving.  dptq_qlinear_static serves them from one fixed
+array compiled into the library.  It runs the same two kernels as dptq_qlinear's
+two-launch path, which gives the same bits as its one-launch path, so its output must be
+bit-identical to dptq_qlinear's.  This file is collected last, so a failure here comes
+after every other test has run; it also passes on its own in a fresh process.
 """
 import ctypes
 
 import pytest
 
-import parity
 from paper_2606_12487_gb300 import inputs
 
 torch = pytest.importorskip("torch")
@@ -36,8 +37,14 @@ def _static_call(dp, layer, x, bits, out):
     return st, lib.dptq_last_error_message().decode()
 
 
+def _device_error(dp):
+    """Status of dptq_last_device_error, which also reads the fixed array's error word."""
+    return dp.load().dptq_last_device_error(None)
+
+
 @pytest.mark.parametrize("M,N,K,B,bits", [(32, 4096, 4096, 4096, 4), (1, 4096, 4096, 4096, 8),
-                                          (17, 1024, 11008, 256, 4), (32, 12288, 4096, 4096, 8)])
+                                          (17, 1024, 11008, 256, 4), (32, 12288, 4096, 4096, 8),
+                                          (5, 272, 2560, 2048, 8), (32, 512, 2560, 2048, 4)])
 def test_static_scratch_matches_qlinear_twice(dp, M, N, K, B, bits):
     wl = inputs.llama2_7b_decode()
     x = torch.from_numpy(inputs.activations(wl, M, K)).cuda()
@@ -50,9 +57,33 @@ def test_static_scratch_matches_qlinear_twice(dp, M, N, K, B, bits):
         st, msg = _static_call(dp, layer, x, bits, out)
         assert st == 0, msg
         torch.cuda.synchronize()
-        parity.check_out(out.cpu().numpy(), ref.cpu().numpy())
-    dp.dptq_last_device_error()
+        assert torch.equal(out.view(torch.int16), ref.view(torch.int16)), "static output differs from dptq_qlinear"
+        assert _device_error(dp) == 0, "a bounded wait gave up inside the static call"
     layer.close()
+
+
+def test_static_call_allocates_no_device_memory(dp):
+    """After one warm-up call (which looks the array up), a call on a new shape leaves
+    the device's free memory unchanged."""
+    wl = inputs.llama2_7b_decode()
+    layers, xs, outs = [], [], []
+    for (M, N, K, B) in [(8, 1024, 4096, 4096), (31, 2048, 2560, 2048)]:
+        layers.append(dp.dptq_pack_weights(torch.from_numpy(inputs.weights(N, K, layer=6)).cuda(), B))
+        xs.append(torch.from_numpy(inputs.activations(wl, M, K)).cuda())
+        outs.append(torch.empty((M, N), dtype=torch.float16, device="cuda"))
+    st, msg = _static_call(dp, layers[0], xs[0], 4, outs[0])
+    assert st == 0, msg
+    torch.cuda.synchronize()
+    free0, _ = torch.cuda.mem_get_info()
+    for bits in (8, 4):
+        st, msg = _static_call(dp, layers[1], xs[1], bits, outs[1])
+        assert st == 0, msg
+    torch.cuda.synchronize()
+    free1, _ = torch.cuda.mem_get_info()
+    assert free1 == free0, f"free device memory changed by {free0 - free1} bytes"
+    assert _device_error(dp) == 0
+    for layer in layers:
+        layer.close()
 
 
 def test_static_scratch_rejects_shapes_beyond_its_limit(dp):
@@ -68,3 +99,5 @@ def test_static_scratch_rejects_shapes_beyond_its_limit(dp):
     out2 = torch.empty((4, 128), dtype=torch.float16, device="cuda")
     st, msg = _static_call(dp, layer2, x2, 4, out2)
     assert st == 2 and "16384" in msg
+    layer.close()
+    layer2.close()
