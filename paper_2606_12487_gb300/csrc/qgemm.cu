@@ -157,13 +157,16 @@ struct Smem {
   __device__ __forceinline__ uint8_t* end(int S) const { return slot(S); }
 };
 
-// FUSED (decode, two-block stages): the launch first rotates and quantizes the token
-// rows itself.  The converter warps of CTA c handle rows c, c + G, ... and publish them
-// on a grid counter; every producer streams its first weight stages meanwhile and
-// requests activation tiles once all M_pad rows are in; the epilogue reads the token
-// scales after the same point.  The last CTA to finish resets the counters.
-template <int NT, int KPS, bool FUSED>
+// RQV != 0 (decode, two-block stages) makes the launch FUSED: it first rotates and
+// quantizes the token rows itself.  Each row is split into rq_np parts (RQV = 16 / rq_np
+// values per chunk and thread: 4 with four parts, 8 with two), and the converter warps
+// of CTA c handle the (row, part) items c, c + G, ... and publish them on a grid counter;
+// every producer streams its first weight stages meanwhile and requests activation tiles
+// once all items are in; the epilogue reads the token scales after the same point.  The
+// last CTA to finish resets the counters.
+template <int NT, int KPS, int RQV>
 __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a) {
+  constexpr bool FUSED = RQV != 0;
   // Two-block stages (token tiles of up to 64, weight streaming) and 192-token tiles
   // widen the weights straight into tensor memory and feed the MMA's A operand from
   // there; other one-block stages widen into shared memory.
@@ -487,7 +490,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
       int nitems = 0;
       for (int item = blockIdx.x; item < a.rq_items; item += gridDim.x) {
         if (nitems) csync();   // the previous item's readers are done with the scratch
-        rotate_quant_row_part(a.rq, item / a.rq_np, item % a.rq_np, a.rq_np, rot_smem, ctid, csync);
+        // Four parts: rows of up to four 4096-element chunks; two parts: up to two.
+        constexpr int kMaxChunks = RQV == 4 ? 4 : 2;
+        rotate_quant_row_part_fast<RQV == 4 ? 4 : 8, kMaxChunks>(a.rq, item / a.rq_np, item % a.rq_np, rot_smem,
+                                                                 ctid, csync);
         ++nitems;
       }
       if (ctid == 0) {
@@ -1015,18 +1021,30 @@ bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan, i
   a.l2_prefetch = (nt <= 64 && m_tiles == 1 && l2_prefetch_allowed()) ? 512LL * 1024 : 0;
   a.rq = RQArgs{};
   a.gsync = nullptr;
-  // Fused: up to 4 CTAs share each token row (each converts and writes a quarter of it),
-  // as long as every part has a CTA of its own.
-  int np = fused ? 4 : 1;
-  while (np > 1 && (long long)M_pad * np > G) np >>= 1;
+  // Fused: every token row is split into 4 parts (each quantizes and writes a quarter of
+  // it) when each part gets a CTA of its own; else into 2 parts with a CTA each, for rows
+  // of at most two 4096-element chunks; else into 4 parts with at most two per CTA.  A
+  // launch whose grid is smaller than that leaves the rows to the separate
+  // rotate-quantize launch (no fused plan).
+  int np = 1;
+  if (fused) {
+    if ((long long)M_pad * 4 <= G)
+      np = 4;
+    else if ((long long)M_pad * 2 <= G && K_pad <= 2 * 4096)
+      np = 2;
+    else if ((long long)M_pad * 4 <= 2LL * G)
+      np = 4;
+    else
+      return false;
+  }
   a.rq_np = np;
   a.rq_items = fused ? M_pad * np : 0;
   return true;
 }
 
-template <int NT, int KPS, bool FUSED = false>
+template <int NT, int KPS, int RQV = 0>
 static cudaError_t launch_nt(const GemmPlan& plan, cudaStream_t s, bool pdl) {
-  cudaError_t e = cudaFuncSetAttribute(qgemm_kernel<NT, KPS, FUSED>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  cudaError_t e = cudaFuncSetAttribute(qgemm_kernel<NT, KPS, RQV>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        plan.smem_bytes);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
@@ -1039,15 +1057,17 @@ static cudaError_t launch_nt(const GemmPlan& plan, cudaStream_t s, bool pdl) {
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = (pdl && pdl_allowed()) ? 1 : 0;
-  return cudaLaunchKernelEx(&cfg, qgemm_kernel<NT, KPS, FUSED>, plan.args);
+  return cudaLaunchKernelEx(&cfg, qgemm_kernel<NT, KPS, RQV>, plan.args);
 }
 
 cudaError_t launch_gemm(const GemmPlan& plan, cudaStream_t s, bool pdl) {
   if (plan.fused) {
+    const bool four = plan.args.rq_np == 4;
+    if (!four && plan.args.rq_np != 2) return cudaErrorInvalidValue;
     switch (plan.nt) {
-      case 16: return launch_nt<16, 2, true>(plan, s, pdl);
-      case 32: return launch_nt<32, 2, true>(plan, s, pdl);
-      case 64: return launch_nt<64, 2, true>(plan, s, pdl);
+      case 16: return four ? launch_nt<16, 2, 4>(plan, s, pdl) : launch_nt<16, 2, 8>(plan, s, pdl);
+      case 32: return four ? launch_nt<32, 2, 4>(plan, s, pdl) : launch_nt<32, 2, 8>(plan, s, pdl);
+      case 64: return four ? launch_nt<64, 2, 4>(plan, s, pdl) : launch_nt<64, 2, 8>(plan, s, pdl);
       default: return cudaErrorInvalidValue;
     }
   }

@@ -472,18 +472,42 @@ __device__ __forceinline__ int rq_pos(int layout, int t, int e) {
   return layout == 2 ? 256 * e + t : layout == 1 ? 256 * (t >> 4) + 16 * e + (t & 15) : 16 * t + e;
 }
 
-// The exact butterflies of one chunk (elements c0 .. c0 + len - 1 of the row at `src`),
-// the same arithmetic as rotate_quant_row; returns the layout f[] ends in.
+// Raw fp16 words of thread `tid`'s 16 consecutive values of the chunk at c0 (round A
+// layout, i = 16 tid + e); zeros past the chunk's length.
+__device__ __forceinline__ void rq_load16(const uint4* src, int c0, int len, int tid, uint4 (&u)[2]) {
+  const int i0 = tid * 16;
+  if (i0 < len) {
+    u[0] = src[(c0 + i0) / 8];
+    u[1] = src[(c0 + i0) / 8 + 1];
+  } else {
+    u[0] = make_uint4(0u, 0u, 0u, 0u);
+    u[1] = u[0];
+  }
+}
+
+// The 16 raw fp16 values to exact fixed point, with the randomized-Hadamard signs.
+__device__ __forceinline__ void rq_fix16(const RQArgs& a, const uint4 (&u)[2], int c0, int len, int tid,
+                                         long long (&f)[16]) {
+  const uint32_t w[8] = {u[0].x, u[0].y, u[0].z, u[0].w, u[1].x, u[1].y, u[1].z, u[1].w};
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+    f[2 * k] = half_to_fixed(w[k] & 0xFFFFu);
+    f[2 * k + 1] = half_to_fixed(w[k] >> 16);
+  }
+  if (a.signs != nullptr && tid * 16 < len) apply_signs(a.signs + c0 + tid * 16, f);
+}
+
+// The exact butterflies of one chunk (elements c0 .. c0 + len - 1 of the row), starting
+// from f[] in the round A layout; returns the layout f[] ends in (see rq_pos).
 template <class Sync>
-__device__ __forceinline__ int rq_chunk(const RQArgs& a, const uint4* src, int c0, int len, int tail_start,
-                                        long long (&f)[16], long long* sx, int tid, Sync sync) {
+__device__ __forceinline__ int rq_bfly(const RQArgs& a, int c0, int len, int tail_start, long long (&f)[16],
+                                       long long* sx, int tid, Sync sync) {
   unsigned long long* const tr = DPTQ_TRACE_BUF();
   (void)tr;
 #define RQC_T(slot) \
   do {              \
     if (tid == 0 && c0 == 0) DPTQ_TRACE_CLOCK(tr, slot); \
   } while (0)
-  RQC_T(170);
   auto lg = [&](int i) { return (c0 + i < tail_start) ? a.log2B : a.log2T; };
   auto bfly = [&](int h) {
 #pragma unroll
@@ -495,21 +519,6 @@ __device__ __forceinline__ int rq_chunk(const RQArgs& a, const uint4* src, int c
       }
   };
   const int i0 = tid * 16;
-  if (i0 < len) {
-    const uint4 u0 = src[(c0 + i0) / 8];
-    const uint4 u1 = src[(c0 + i0) / 8 + 1];
-    const uint32_t w[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
-#pragma unroll
-    for (int k = 0; k < 8; ++k) {
-      f[2 * k] = half_to_fixed(w[k] & 0xFFFFu);
-      f[2 * k + 1] = half_to_fixed(w[k] >> 16);
-    }
-    if (a.signs != nullptr) apply_signs(a.signs + c0 + i0, f);
-  } else {
-#pragma unroll
-    for (int k = 0; k < 16; ++k) f[k] = 0;
-  }
-  if (tid == 0 && c0 == 0) { volatile long long sink = f[0] ^ f[15]; (void)sink; }
   RQC_T(171);
   {
     const int L = lg(i0 < len ? i0 : 0);
@@ -524,7 +533,6 @@ __device__ __forceinline__ int rq_chunk(const RQArgs& a, const uint4* src, int c
         if (bit < L) bfly(1 << bit);
     }
   }
-  if (tid == 0 && c0 == 0) { volatile long long sink = f[0] ^ f[15]; (void)sink; }
   RQC_T(172);
   const int maxlg = (c0 + len > tail_start) ? max(a.log2B, a.log2T) : a.log2B;
   if (maxlg <= 4) return 0;
@@ -535,7 +543,6 @@ __device__ __forceinline__ int rq_chunk(const RQArgs& a, const uint4* src, int c
   const int iB = 256 * (tid >> 4) + (tid & 15);
 #pragma unroll
   for (int e = 0; e < 16; ++e) f[e] = sx[pad_idx(iB + 16 * e)];
-  if (tid == 0 && c0 == 0) { volatile long long sink = f[0] ^ f[15]; (void)sink; }
   RQC_T(173);
   {
     const int L = lg(iB);
@@ -550,7 +557,6 @@ __device__ __forceinline__ int rq_chunk(const RQArgs& a, const uint4* src, int c
         if (bit < L) bfly(1 << (bit - 4));
     }
   }
-  if (tid == 0 && c0 == 0) { volatile long long sink = f[0] ^ f[15]; (void)sink; }
   RQC_T(174);
   if (maxlg <= 8) return 1;
 #pragma unroll
@@ -558,7 +564,6 @@ __device__ __forceinline__ int rq_chunk(const RQArgs& a, const uint4* src, int c
   sync();
 #pragma unroll
   for (int e = 0; e < 16; ++e) f[e] = sx[pad_idx(256 * e + tid)];
-  if (tid == 0 && c0 == 0) { volatile long long sink = f[0] ^ f[15]; (void)sink; }
   RQC_T(175);
   if (c0 + len <= tail_start && a.log2B == 12) {
     bfly(1);
@@ -582,41 +587,58 @@ __device__ __forceinline__ int rq_chunk(const RQArgs& a, const uint4* src, int c
         }
     }
   }
-  if (tid == 0 && c0 == 0) { volatile long long sink = f[0] ^ f[15]; (void)sink; }
   RQC_T(176);
 #undef RQC_T
   return 2;
+}
+
+// Load, fix and butterflies of one chunk: the same arithmetic as rotate_quant_row.
+template <class Sync>
+__device__ __forceinline__ int rq_chunk(const RQArgs& a, const uint4* src, int c0, int len, int tail_start,
+                                        long long (&f)[16], long long* sx, int tid, Sync sync) {
+  uint4 u[2];
+  rq_load16(src, c0, len, tid, u);
+  rq_fix16(a, u, c0, len, tid, f);
+  return rq_bfly(a, c0, len, tail_start, f, sx, tid, sync);
 }
 
 __device__ __forceinline__ uint32_t e4m3_byte(float v) { return e4m3x2(v, 0.f) & 0xFFu; }
 
 static_assert(kRQPartSmemBytes == kChunkPadded * 8 + 2 * kChunk + 16 * 8, "part scratch layout");
 
-// The share `part` of `np` (1, 2 or 4) of one row in the fused decode launch, writing
-// the GEMM operand planes (kRQAct layout) and, for part 0, the row's scale.  Every part
-// runs the row's butterflies (cheap), and takes the absmax from the largest |S| of each
-// block size: the conversion to fp32 is odd and monotone in S, so max|y| is the
-// conversion of max|S|.  It then converts, quantizes and writes only the values whose
-// index e (in the final layout) lies in [16 part / np, 16 (part + 1) / np), staging the
-// codes in shared memory for coalesced 32-bit stores.  Rows of more than one chunk run
-// the butterflies twice (the values are not kept).  Codes and scales equal those of
-// rotate_quant_row<kRQAct>.  smem: kRQPartSmemBytes, 16-byte aligned; 256 threads meet
-// at sync(); the caller synchronizes before reusing smem for another row.
-template <class Sync>
-__device__ __forceinline__ void rotate_quant_row_part(const RQArgs& a, int row, int part, int np,
-                                                      unsigned char* smem, int tid, Sync sync) {
+// The share `part` of 16 / VPC parts of one row in the fused decode launch, for rows of
+// at most MAXCH chunks (K <= 4096 MAXCH; VPC * MAXCH <= 16): the codes and scale of
+// rotate_quant_row<kRQAct>, computed for low latency rather than throughput.
+//   * The next chunk's 32 bytes per thread are requested before the current chunk's
+//     butterflies run, so the row's global loads overlap the arithmetic.
+//   * The VPC values of each chunk that this part quantizes are converted to fp32 as the
+//     chunk finishes and stay in registers (at most 16), so no butterflies are redone.
+//   * The row absmax: each thread converts its largest |S| of each block size once (the
+//     conversion is odd and monotone, so the fp32 of the largest |S| is the largest |y|);
+//     the warp maximum is one redux on the fp32 bit patterns (non-negative floats order as
+//     their bits), then one shared-memory step across the 8 warps.
+//   * All of the part's codes are staged in shared memory (the transpose buffer, free once
+//     the butterflies are done) and stored after one barrier, as 32-bit words whose four
+//     codes are consecutive in k.
+// smem: kRQPartSmemBytes, 16-byte aligned; 256 threads meet at sync(); the caller
+// synchronizes before reusing smem.
+template <int VPC, int MAXCH, class Sync>
+__device__ __forceinline__ void rotate_quant_row_part_fast(const RQArgs& a, int row, int part, unsigned char* smem,
+                                                           int tid, Sync sync) {
+  static_assert(VPC == 4 || VPC == 8, "a part quantizes 4 or 8 values of each chunk per thread");
+  static_assert(VPC * MAXCH <= 16, "at most 16 kept values per thread");
+  constexpr int NP = 16 / VPC;
   long long* sx = reinterpret_cast<long long*>(smem);
-  uint8_t* cst = smem + (size_t)kChunkPadded * 8;                 // [2][kChunk] staged E4M3 codes
-  long long* red = reinterpret_cast<long long*>(cst + 2 * kChunk);   // [16] warp maxima
+  uint8_t* stg = smem;   // [planes][K_pad] staged codes, in sx once its readers are done
+  float* redf = reinterpret_cast<float*>(smem + (size_t)kChunkPadded * 8 + 2 * kChunk);   // [8] warp maxima
   unsigned long long* const tr = DPTQ_TRACE_BUF();
   (void)tr;
   const int K = a.K;
   const int K_pad = a.KB * 128;
-  const bool live = row < a.rows_in;
   const int tail_start = a.nfull << a.log2B;
   const int bits = a.bits;
-  const int qmax = (1 << (bits - 1)) - 1;
-  const float qmaxf = (float)qmax, qminf = (float)(-(1 << (bits - 1)));
+  const int nch = (K + kChunk - 1) / kChunk;   // 1..MAXCH
+  const int e0 = part * VPC;                   // this part's values: e in [e0, e0 + VPC)
   uint8_t* act = static_cast<uint8_t*>(a.out);
   const size_t plane_stride = (size_t)a.KB * a.rows_out * 128;
   auto store4 = [&](int k, uint32_t w0, uint32_t w1) {   // codes k .. k + 3 (k % 4 == 0)
@@ -626,167 +648,142 @@ __device__ __forceinline__ void rotate_quant_row_part(const RQArgs& a, int row, 
     if (bits == 8) *reinterpret_cast<uint32_t*>(act + plane_stride + off) = w1;
   };
 
-  if (!live) {   // padding row: zero codes (words split evenly over the parts) and scale
+  if (row >= a.rows_in) {   // padding row: zero codes (words split evenly over the parts) and scale
     const int W = K_pad / 4;
-    for (int w = W * part / np + tid; w < W * (part + 1) / np; w += kRQThreads) store4(4 * w, 0u, 0u);
+    for (int w = W * part / NP + tid; w < W * (part + 1) / NP; w += kRQThreads) store4(4 * w, 0u, 0u);
     if (part == 0 && tid == 0 && a.scales != nullptr) a.scales[row] = 0.f;
     return;
   }
-
+  if (tid == 0) DPTQ_TRACE_CLOCK(tr, 160 + 10);
   const uint4* src = reinterpret_cast<const uint4*>(a.x + (size_t)row * K);
-  long long f[16];
-  int L0 = 0;
-  // With 4 parts and at most 3 chunks, each chunk's 4 values of this part are converted
-  // to fp32 in pass 1 (the conversion does not depend on the scale) and stay in
-  // registers (kept[chunk]) for pass 2; otherwise pass 2 repeats the butterflies.
-  const bool keep = np == 4 && K <= 3 * kChunk;
-  float kept[3][4];
-  int kept_L[3] = {0, 0, 0};
-  // ---- pass 1: butterflies, largest |S| per block size
+  float kept[MAXCH][VPC];
+  int kept_L[MAXCH];
   long long mB = 0, mT = 0;
-  for (int c0 = 0; c0 < K; c0 += kChunk) {
-    const int len = min(kChunk, K - c0);
-    const int L = rq_chunk(a, src, c0, len, tail_start, f, sx, tid, sync);
-    L0 = L;
-    if (keep) {
-      long long w[4];
-      switch (part) {
-        case 0: w[0] = f[0]; w[1] = f[1]; w[2] = f[2]; w[3] = f[3]; break;
-        case 1: w[0] = f[4]; w[1] = f[5]; w[2] = f[6]; w[3] = f[7]; break;
-        case 2: w[0] = f[8]; w[1] = f[9]; w[2] = f[10]; w[3] = f[11]; break;
-        default: w[0] = f[12]; w[1] = f[13]; w[2] = f[14]; w[3] = f[15]; break;
-      }
-      float v[4];
+  uint4 u[2];
+  rq_load16(src, 0, min(kChunk, K), tid, u);
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const int i = rq_pos(L, tid, 4 * part + j);
-        v[j] = i < len ? fixed_to_rotated(w[j], (c0 + i < tail_start) ? a.log2B : a.log2T, a.c_hi, a.c_lo) : 0.f;
-      }
-      switch (c0 / kChunk) {
-#define RQ_KEEP(n)                                                            \
-  case n:                                                                     \
-    kept[n][0] = v[0]; kept[n][1] = v[1]; kept[n][2] = v[2]; kept[n][3] = v[3]; \
-    kept_L[n] = L;                                                            \
-    break;
-        RQ_KEEP(0)
-        RQ_KEEP(1)
-        default:
-          kept[2][0] = v[0]; kept[2][1] = v[1]; kept[2][2] = v[2]; kept[2][3] = v[3];
-          kept_L[2] = L;
-          break;
-#undef RQ_KEEP
-      }
-    }
-    if (len == kChunk && c0 + len <= tail_start) {   // every value is in a block of size B
+  for (int c = 0; c < MAXCH; ++c) {
+    kept_L[c] = 0;
+    if (c < nch) {
+      const int c0 = c * kChunk;
+      const int len = min(kChunk, K - c0);
+      long long f[16];
+      rq_fix16(a, u, c0, len, tid, f);
+      if (c + 1 < nch) rq_load16(src, c0 + kChunk, min(kChunk, K - c0 - kChunk), tid, u);
+      const int L = rq_bfly(a, c0, len, tail_start, f, sx, tid, sync);
+      kept_L[c] = L;
+      if (len == kChunk && c0 + len <= tail_start) {   // every value is in a block of size B
 #pragma unroll
-      for (int e = 0; e < 16; ++e) {
-        const long long v = f[e] < 0 ? -f[e] : f[e];
-        mB = v > mB ? v : mB;
-      }
-    } else {
-#pragma unroll
-      for (int e = 0; e < 16; ++e) {
-        const int i = rq_pos(L, tid, e);
-        if (i < len) {
+        for (int e = 0; e < 16; ++e) {
           const long long v = f[e] < 0 ? -f[e] : f[e];
-          if (c0 + i < tail_start)
-            mB = v > mB ? v : mB;
-          else
-            mT = v > mT ? v : mT;
+          mB = v > mB ? v : mB;
         }
+      } else {
+#pragma unroll
+        for (int e = 0; e < 16; ++e) {
+          const int i = rq_pos(L, tid, e);
+          const long long v = f[e] < 0 ? -f[e] : f[e];
+          if (i < len) {
+            if (c0 + i < tail_start)
+              mB = v > mB ? v : mB;
+            else
+              mT = v > mT ? v : mT;
+          }
+        }
+      }
+      long long v[VPC];   // f[e0 .. e0 + VPC - 1]; `part` is uniform over the CTA
+      if constexpr (VPC == 4) {
+        switch (part) {
+          case 0: v[0] = f[0]; v[1] = f[1]; v[2] = f[2]; v[3] = f[3]; break;
+          case 1: v[0] = f[4]; v[1] = f[5]; v[2] = f[6]; v[3] = f[7]; break;
+          case 2: v[0] = f[8]; v[1] = f[9]; v[2] = f[10]; v[3] = f[11]; break;
+          default: v[0] = f[12]; v[1] = f[13]; v[2] = f[14]; v[3] = f[15]; break;
+        }
+      } else {
+        if (part == 0) {
+#pragma unroll
+          for (int j = 0; j < 8; ++j) v[j] = f[j];
+        } else {
+#pragma unroll
+          for (int j = 0; j < 8; ++j) v[j] = f[8 + j];
+        }
+      }
+#pragma unroll
+      for (int j = 0; j < VPC; ++j) {
+        const int i = rq_pos(L, tid, e0 + j);
+        kept[c][j] = i < len ? fixed_to_rotated(v[j], (c0 + i < tail_start) ? a.log2B : a.log2T, a.c_hi, a.c_lo)
+                             : 0.f;
       }
     }
   }
   if (tid == 0) DPTQ_TRACE_CLOCK(tr, 140);
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const long long b = __shfl_xor_sync(0xffffffffu, mB, o), t = __shfl_xor_sync(0xffffffffu, mT, o);
-    mB = b > mB ? b : mB;
-    mT = t > mT ? t : mT;
-  }
-  if ((tid & 31) == 0) {
-    red[tid >> 5] = mB;
-    red[8 + (tid >> 5)] = mT;
-  }
-  sync();
-#pragma unroll
-  for (int w = 0; w < kRQThreads / 32; ++w) {
-    mB = red[w] > mB ? red[w] : mB;
-    mT = red[8 + w] > mT ? red[8 + w] : mT;
-  }
+  // Row absmax (see above); the barrier also ends every read of sx.
   const float yB = mB ? fixed_to_rotated(mB, a.log2B, a.c_hi, a.c_lo) : 0.f;
   const float yT = mT ? fixed_to_rotated(mT, a.log2T, a.c_hi, a.c_lo) : 0.f;
-  const float amax = fmaxf(yB, yT);
+  const uint32_t wmax = __reduce_max_sync(0xffffffffu, __float_as_uint(fmaxf(yB, yT)));
+  if ((tid & 31) == 0) redf[tid >> 5] = __uint_as_float(wmax);
+  sync();
+  float amax = redf[0];
+#pragma unroll
+  for (int w = 1; w < kRQThreads / 32; ++w) amax = fmaxf(amax, redf[w]);
+  const int qmax = (1 << (bits - 1)) - 1;
+  const float qmaxf = (float)qmax, qminf = (float)(-(1 << (bits - 1)));
   const float s = __fdiv_rn(amax, qmaxf);
   const bool nz = amax > 0.f;
   const float rs = nz ? __frcp_rn(s) : 0.f;
   if (part == 0 && tid == 0 && a.scales != nullptr) a.scales[row] = nz ? s : 0.f;
   if (tid == 0) DPTQ_TRACE_CLOCK(tr, 141);
 
-  // ---- pass 2: this part's codes, chunk by chunk
-  const int elo = 16 * part / np, ehi = 16 * (part + 1) / np;
-  for (int c0 = 0; c0 < K; c0 += kChunk) {
-    const int len = min(kChunk, K - c0);
-    const int ch = c0 / kChunk;
-    int L = L0;
-    if (keep)
-      L = ch == 0 ? kept_L[0] : ch == 1 ? kept_L[1] : kept_L[2];
-    else if (K > kChunk)
-      L = rq_chunk(a, src, c0, len, tail_start, f, sx, tid, sync);
-#pragma unroll 1
-    for (int g4 = elo >> 2; g4 < ehi >> 2; ++g4) {   // this part's values, 4 at a time
-      int idx[4];
-      float y[4], c[4] = {0.f, 0.f, 0.f, 0.f};
+  // Codes of this part, staged at their k (plane 0 at stg[k], plane 1 at stg[K_pad + k]).
 #pragma unroll
-      for (int j = 0; j < 4; ++j) idx[j] = rq_pos(L, tid, 4 * g4 + j);
-      if (keep) {
-        switch (ch) {
-          case 0: y[0] = kept[0][0]; y[1] = kept[0][1]; y[2] = kept[0][2]; y[3] = kept[0][3]; break;
-          case 1: y[0] = kept[1][0]; y[1] = kept[1][1]; y[2] = kept[1][2]; y[3] = kept[1][3]; break;
-          default: y[0] = kept[2][0]; y[1] = kept[2][1]; y[2] = kept[2][2]; y[3] = kept[2][3]; break;
-        }
-      } else {
-        long long v[4];
-        switch (g4) {
-          case 0: v[0] = f[0]; v[1] = f[1]; v[2] = f[2]; v[3] = f[3]; break;
-          case 1: v[0] = f[4]; v[1] = f[5]; v[2] = f[6]; v[3] = f[7]; break;
-          case 2: v[0] = f[8]; v[1] = f[9]; v[2] = f[10]; v[3] = f[11]; break;
-          default: v[0] = f[12]; v[1] = f[13]; v[2] = f[14]; v[3] = f[15]; break;
-        }
+  for (int c = 0; c < MAXCH; ++c) {
+    if (c < nch) {
+      const int c0 = c * kChunk;
+      const int len = min(kChunk, K - c0);
+      const int L = kept_L[c];
 #pragma unroll
-        for (int j = 0; j < 4; ++j)
-          y[j] = idx[j] < len ? fixed_to_rotated(v[j], (c0 + idx[j] < tail_start) ? a.log2B : a.log2T, a.c_hi, a.c_lo)
-                              : 0.f;
-      }
-      if (nz) quant_code4(y, s, rs, qminf, qmaxf, c);
+      for (int g4 = 0; g4 < VPC / 4; ++g4) {
+        float y[4] = {kept[c][4 * g4], kept[c][4 * g4 + 1], kept[c][4 * g4 + 2], kept[c][4 * g4 + 3]};
+        float q[4] = {0.f, 0.f, 0.f, 0.f};
+        if (nz) quant_code4(y, s, rs, qminf, qmaxf, q);
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        if (idx[j] < len) {
-          if (bits == 4) {
-            cst[idx[j]] = (uint8_t)e4m3_byte(c[j]);
-          } else {
-            const float m = fabsf(c[j]);
-            const float h = __fmul_rn(floorf(__fmul_rn(m, 0.0625f)), 16.f);
-            cst[idx[j]] = (uint8_t)e4m3_byte(__fadd_rn(copysignf(h, c[j]), 0.0f));
-            cst[kChunk + idx[j]] = (uint8_t)e4m3_byte(__fadd_rn(copysignf(__fsub_rn(m, h), c[j]), 0.0f));
+        for (int j = 0; j < 4; ++j) {
+          const int i = rq_pos(L, tid, e0 + 4 * g4 + j);
+          if (i < len) {
+            if (bits == 4) {
+              stg[c0 + i] = (uint8_t)e4m3_byte(q[j]);
+            } else {
+              const float m = fabsf(q[j]);
+              const float h = __fmul_rn(floorf(__fmul_rn(m, 0.0625f)), 16.f);
+              stg[c0 + i] = (uint8_t)e4m3_byte(__fadd_rn(copysignf(h, q[j]), 0.0f));
+              stg[K_pad + c0 + i] = (uint8_t)e4m3_byte(__fadd_rn(copysignf(__fsub_rn(m, h), q[j]), 0.0f));
+            }
           }
         }
       }
     }
-    if (tid == 0 && c0 == 0) DPTQ_TRACE_CLOCK(tr, 142);
-    sync();
-    for (int w = tid; w < len / 4; w += kRQThreads) {
-      const int i = 4 * w;
-      const int ei = L == 2 ? i >> 8 : L == 1 ? (i >> 4) & 15 : i & 15;
-      if (ei >= elo && ei < ehi)
-        store4(c0 + i, *reinterpret_cast<const uint32_t*>(cst + i),
-               *reinterpret_cast<const uint32_t*>(cst + kChunk + i));
-    }
-    if (tid == 0 && c0 == 0) DPTQ_TRACE_CLOCK(tr, 143);
-    sync();   // the staging buffer is reused by the next chunk
   }
-  if (part == np - 1)   // k in [K, K_pad): zero codes
+  if (tid == 0) DPTQ_TRACE_CLOCK(tr, 142);
+  sync();
+  // The words whose values this part owns: value index of element i in layout L.
+#pragma unroll
+  for (int c = 0; c < MAXCH; ++c) {
+    if (c < nch) {
+      const int c0 = c * kChunk;
+      const int len = min(kChunk, K - c0);
+      const int L = kept_L[c];
+      for (int w = tid; w < len / 4; w += kRQThreads) {
+        const int i = 4 * w;
+        const int ei = L == 2 ? i >> 8 : L == 1 ? (i >> 4) & 15 : i & 15;
+        if (ei >= e0 && ei < e0 + VPC)
+          store4(c0 + i, *reinterpret_cast<const uint32_t*>(stg + c0 + i),
+                 *reinterpret_cast<const uint32_t*>(stg + K_pad + c0 + i));
+      }
+    }
+  }
+  if (part == NP - 1)   // k in [K, K_pad): zero codes
     for (int k = K + 4 * tid; k < K_pad; k += 4 * kRQThreads) store4(k, 0u, 0u);
+  if (tid == 0) DPTQ_TRACE_CLOCK(tr, 143);
 }
 
 }  // namespace dptq

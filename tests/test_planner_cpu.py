@@ -84,12 +84,26 @@ def test_fused_decode_plans(N, K, M, bits):
         with pytest.raises(dptq.DptqError):
             dptq.dptq_plan_info(M, N, K, bits, 152, fused=True)
         return
+    split = dptq.dptq_plan_info(M, N, K, bits, 152)
+    M_pad, G = split["M_pad"], split["grid"]
+    if M_pad * 4 > 2 * G and (M_pad * 2 > G or K > 8192):
+        # too few CTAs for the rows' parts: dptq_qlinear takes the two-launch path
+        with pytest.raises(dptq.DptqError):
+            dptq.dptq_plan_info(M, N, K, bits, 152, fused=True)
+        return
     p = dptq.dptq_plan_info(M, N, K, bits, 152, fused=True)
     _check_plan(p, M, N, K, bits, 152)
     assert p["fused"] == 1 and p["kps"] == 2 and p["nt"] <= 64 and p["stages"] >= 3
     assert p["smem_bytes"] <= SMEM_LIMIT
-    # each token row is split over rq_np CTAs, each part with a CTA of its own
-    assert p["rq_np"] in (1, 2, 4) and (p["rq_np"] == 1 or p["M_pad"] * p["rq_np"] <= p["grid"])
+    # each token row is split into 4 parts, each with a CTA of its own; else into 2 parts
+    # (rows of at most two 4096-element chunks); else 4 parts with at most two per CTA
+    np_ = p["rq_np"]
+    assert np_ in (2, 4)
+    if np_ == 2:
+        assert M_pad * 4 > p["grid"] and M_pad * 2 <= p["grid"] and K <= 8192
+    else:
+        assert M_pad * 4 <= 2 * p["grid"]
+        assert M_pad * 4 <= p["grid"] or M_pad * 2 > p["grid"] or K > 8192
 
 
 def test_fused_plan_refused_beyond_64_tokens():
