@@ -207,7 +207,10 @@ class Stack:
         return 2 * self.M * N * K
 
     def step_launches(self):
-        return (1 if self.path == "fused" else 2) * len(self.groups) * len(self.layers)
+        """Kernel launches of one step: dptq_qlinear is one launch up to 64 tokens (fused)
+        and two above (rotate-quantize, then GEMM); the split path is always two."""
+        per = 1 if (self.path == "fused" and self.M <= 64) else 2
+        return per * len(self.groups) * len(self.layers)
 
     def h2d_bytes(self):
         return sum(x.numel() * 2 for x in self.x)
@@ -317,7 +320,9 @@ def measure_gemm_kernels(stack, stream):
 
 def e2e_measure(stack, g, stream, steps, world):
     """Same metric through the public API with host buffers: per step, H2D copies of
-    the step's inputs from pinned memory, the stack, and a D2H read of the result."""
+    the step's inputs from pinned memory, the stack as the user calls it (every
+    projection a dptq_qlinear call through the C ABI, launched eagerly, no graph), and a
+    D2H read of the result."""
     import torch
     hx = [x.cpu().pin_memory() for x in stack.x]
     hout = torch.empty(stack.out[-1].shape, dtype=torch.float16).pin_memory()
@@ -325,8 +330,7 @@ def e2e_measure(stack, g, stream, steps, world):
         with torch.cuda.stream(stream):
             for h, d in zip(hx, stack.x):
                 d.copy_(h, non_blocking=True)
-        g.replay()
-        with torch.cuda.stream(stream):
+            stack.run(stream)
             hout.copy_(stack.out[-1], non_blocking=True)
     torch.cuda.synchronize()
     barrier(world)
@@ -338,7 +342,7 @@ def e2e_measure(stack, g, stream, steps, world):
         for _ in range(steps):
             for h, d in zip(hx, stack.x):
                 d.copy_(h, non_blocking=True)
-            g.replay()
+            stack.run(stream)
             hout.copy_(stack.out[-1], non_blocking=True)
         e1.record(stream)
     torch.cuda.synchronize()
@@ -476,6 +480,103 @@ def run_shapes(args):
                                                   ">= 2x L2 of copies", "shapes": rows, "extra_kernels": extra}),
           flush=True)
     return 0
+
+
+# ------------------------------------------------------------------------------ prefill stack
+PREFILL_M = 2048
+
+
+def load_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f)
+    except OSError:
+        return {}
+
+
+def measure_prefill(dptq, device, stream, steps, warmup, world, local):
+    """The LLaMA-3-8B prefill projection stack: 32 layers at M = 2048 tokens with the
+    seeded mask of 6 A8 layers; each projection group (q|k|v, o, gate|up, down) is one
+    dptq_qlinear call, i.e. a rotate-quantize launch and a GEMM launch, and the step is
+    replayed as a CUDA graph.  Inputs (16-59 MB per group) and weights (3.5 GB) exceed
+    L2 between replays.  Returns the `prefill` object of the JSON line."""
+    import torch
+    from paper_2606_12487_gb300 import inputs
+    wl = inputs.llama3_8b_prefill()
+    M = PREFILL_M
+    layers = build_stack(dptq, wl, device)
+    max_k = max(K for _, K, _, _, _ in stack_groups(wl))
+    dptq.dptq_reserve(M, max_k, 0)
+    stack = Stack(dptq, wl, layers, M, device, "fused")
+    g = capture(stack, stream)
+    ms, clocks = time_graph(g, stream, steps, warmup, world, local)
+    ms = max_over_ranks(ms, world, device)
+    ops = sum(2 * M * N * K for _, K, N, _, _ in stack.groups) * len(layers)
+    # One eager step with CUDA events around every launch (on the launching stream): the
+    # GEMM launches and the rotate-quantize launches, timed apart.
+    dptq.dptq_qlinear_quantize(layers[0][0], stack.x[0], 4, stream=stream)
+    torch.cuda.synchronize()
+    t_q = t_g = 0.0
+    gemm_ops = 0
+    evs = []
+    with torch.cuda.stream(stream):
+        for li, hs in enumerate(layers):
+            bits = wl.bits(li)
+            for gi, h in enumerate(hs):
+                e = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+                e[0].record(stream)
+                dptq.dptq_qlinear_quantize(h, stack.x[gi], bits, stream=stream)
+                e[1].record(stream)
+                dptq.dptq_qlinear_gemm(h, M, bits, stack.out[gi], stream=stream)
+                e[2].record(stream)
+                _, K, N, _, _ = stack.groups[gi]
+                evs.append((e, 2 * M * N * K))
+    torch.cuda.synchronize()
+    for e, o in evs:
+        t_q += e[0].elapsed_time(e[1]) / 1e3
+        t_g += e[1].elapsed_time(e[2]) / 1e3
+        gemm_ops += o
+    peaks = load_peaks()
+    bf16_sus = float(peaks.get("bf16_tflops_sustained", 1700.0))
+    bf16_burst = float(peaks.get("bf16_tflops", 1900.0))
+    fp8_sus, fp8_burst = 2.0 * bf16_sus, 2.0 * bf16_burst
+    n_gemm = len(evs)
+    gemm_tops = gemm_ops / t_g / 1e12
+    stack_tops = ops / (ms / 1e3) / 1e12
+    rot_bytes = sum(M * K * 2 + M * K * wl.bits(li) // 8 + 4 * M
+                    for li in range(len(layers)) for _, K, _, _, _ in stack.groups)
+    hbm = float(peaks.get("hbm_gbs", 6800.0))
+    del g
+    out = {
+        "workload": f"llama3-8b prefill projection stack, {len(layers)} layers, M={M} tokens, "
+                    f"A8 on layers {list(wl.mask_a8)}, block Hadamard 2048",
+        "tokens_per_s": aggregate_value(M, world, ms / 1e3), "ms_per_step": ms, "steps": steps, "warmup": warmup,
+        "effective_tops": stack_tops, "ops_per_step": ops,
+        "ops_note": "2*M*N*K effective integer ops per projection (A8 layers issue twice the MMA work)",
+        "gpu_launches": stack.step_launches() * steps,
+        "roofline": {"bound": "tensor", "achieved": stack_tops, "peak": fp8_sus, "unit": "TFLOP/s",
+                     "frac": stack_tops / fp8_sus,
+                     "peak_source": "2 x MEASURED_PEAKS.json bf16_tflops_sustained (fp8 = 2 x bf16 nominal ratio)",
+                     "achieved_note": "effective ops of the step / graph-replay step time (both launches of every "
+                                      "projection)",
+                     "gemm_kernel": {"kernel": "qgemm_kernel (192-token tiles A4, 128-token tiles A8)",
+                                     "achieved_tflops": gemm_tops, "peak": fp8_burst,
+                                     "frac": gemm_tops / fp8_burst, "launches": n_gemm,
+                                     "avg_launch_us": t_g / n_gemm * 1e6,
+                                     "note": "eager pass, CUDA events around each GEMM launch on its stream; "
+                                             "peak = 2 x bf16 burst"}},
+        "time_shares": {"gemm": t_g / (t_g + t_q), "rotate_quantize": t_q / (t_g + t_q)},
+        "rotate_quantize": {"us_per_step": t_q * 1e6, "gbs": rot_bytes / t_q / 1e9,
+                            "hbm_frac": rot_bytes / t_q / 1e9 / hbm,
+                            "bytes_note": "2MK (fp16 in) + MK b/8 (codes) + 4M (scales) per launch"},
+        "clocks": clocks,
+    }
+    for hs in layers:
+        for h in hs:
+            h.close()
+    del stack, layers
+    torch.cuda.synchronize()
+    return out
 
 
 # ------------------------------------------------------------------------------ oracle timing
@@ -652,6 +753,8 @@ def main(argv=None):
                     help="time each decode / prefill projection shape alone and print one JSON line of them")
     ap.add_argument("--extra-only", action="store_true",
                     help="with --shapes: time only the KV4 quantizer and the sensitivity policy")
+    ap.add_argument("--prefill-steps", type=int, default=10,
+                    help="timed steps of the LLaMA-3-8B prefill stack (the `prefill` object; 0 = skip it)")
     ap.add_argument("--only", default="",
                     help="with --shapes: only the shapes whose label 'NAME M=.. A..' contains this text "
                          "(the KV4 and policy timings still follow)")
@@ -687,12 +790,9 @@ def main(argv=None):
     value = aggregate_value(args.m, world, ms_max / 1e3)
 
     tb, to, tt, n_gemm = measure_gemm_kernels(stack, stream)
-    peaks = {}
-    try:
-        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
-            peaks = json.load(f)
-    except OSError:
-        pass
+    n_launches_step = stack.step_launches()
+    h2d_bytes, d2h_bytes = stack.h2d_bytes(), stack.d2h_bytes()
+    peaks = load_peaks()
     hbm_peak = float(peaks.get("hbm_gbs", 6800.0))
     # The timed step is nothing but the n_gemm launches of this kernel, back to back, so
     # its average launch duration over the timed region is the step time / n_gemm and the
@@ -717,6 +817,17 @@ def main(argv=None):
         del gm, st
     sweep[str(args.m)] = {"tokens_per_s": value, "ms_per_step": ms_max, "gemm_gbs": achieved,
                           "isolated_launch_gbs": isolated}
+
+    # Free the decode stack before the prefill stack is packed.
+    del g, stack
+    for hs in layers:
+        for h in hs:
+            h.close()
+    torch.cuda.synchronize()
+    prefill = None
+    if args.prefill_steps > 0 and not args.layers:
+        print(f"[bench] rank {rank}/{world}: prefill stack", file=sys.stderr, flush=True)
+        prefill = measure_prefill(dptq, device, stream, args.prefill_steps, args.warmup, world, local)
 
     dptq.dptq_last_device_error()
     if rank != 0:
@@ -748,11 +859,12 @@ def main(argv=None):
         "stack_weight_gbs": weight_bytes / (ms_max / 1e3) / 1e9,
         "m_sweep": sweep,
         "e2e": {"value": aggregate_value(args.m, world, e2e_s), "unit": UNIT,
-                "h2d_bytes_per_step": stack.h2d_bytes(), "d2h_bytes_per_step": stack.d2h_bytes(),
+                "h2d_bytes_per_step": h2d_bytes, "d2h_bytes_per_step": d2h_bytes,
                 "wall_ms_per_step": e2e_wall_s * 1e3},
-        "gpu_launches": stack.step_launches() * args.steps,
+        "gpu_launches": n_launches_step * args.steps,
         "clocks": clocks,
         "cpu_baseline": cpu,
+        "prefill": prefill,
     }
     print(json.dumps(line), flush=True)
     return 0

@@ -602,13 +602,76 @@ __device__ __forceinline__ int rq_chunk(const RQArgs& a, const uint4* src, int c
   return rq_bfly(a, c0, len, tail_start, f, sx, tid, sync);
 }
 
+// The same butterflies as rq_bfly with a small code footprint, for code that runs once
+// per launch (the fused decode rotation), where every instruction is fetched cold: the
+// three rounds share one body (a transpose through sx between rounds, then the round's
+// four levels on the 16 values in registers), so rounds B and C run from instructions
+// that round A brought into the instruction cache.  Returns the layout f[] ends in.
+template <class Sync>
+__device__ __forceinline__ int rq_bfly_compact(const RQArgs& a, int c0, int len, int tail_start, long long (&f)[16],
+                                            long long* sx, int tid, Sync sync) {
+  const int maxlg = (c0 + len > tail_start) ? max(a.log2B, a.log2T) : a.log2B;
+  const int rounds = maxlg <= 4 ? 1 : maxlg <= 8 ? 2 : 3;
+  // Blocks are B-sized before tail_start and tail-sized after, so only chunks that reach
+  // the tail can mix block sizes.
+  const bool mixed = c0 + len > tail_start && a.log2T != a.log2B;
+#pragma unroll 1
+  for (int r = 0; r < rounds; ++r) {
+    if (r > 0) {
+      sync();   // the previous readers of sx are done
+#pragma unroll
+      for (int e = 0; e < 16; ++e) sx[pad_idx(rq_pos(r - 1, tid, e))] = f[e];
+      sync();
+#pragma unroll
+      for (int e = 0; e < 16; ++e) f[e] = sx[pad_idx(rq_pos(r, tid, e))];
+    }
+    const int base = 4 * r;
+    if (!mixed && a.log2B >= base + 4) {   // every element's block spans the round's 4 levels
+#pragma unroll
+      for (int bit = 0; bit < 4; ++bit) {
+        const int h = 1 << bit;
+#pragma unroll
+        for (int e = 0; e < 16; ++e)
+          if ((e & h) == 0) {
+            const long long p = f[e], q = f[e + h];
+            f[e] = p + q;
+            f[e + h] = p - q;
+          }
+      }
+    } else {
+      // A level applies to an element while it is below the log2 of the element's block.
+#pragma unroll
+      for (int bit = 0; bit < 4; ++bit) {
+        const int lvl = base + bit;
+        const int h = 1 << bit;
+#pragma unroll
+        for (int e = 0; e < 16; ++e) {
+          if ((e & h) == 0) {
+            const int i = rq_pos(r, tid, e);
+            const int lg = (c0 + i < tail_start) ? a.log2B : a.log2T;
+            if (lvl < lg) {
+              const long long p = f[e], q = f[e + h];
+              f[e] = p + q;
+              f[e + h] = p - q;
+            }
+          }
+        }
+      }
+    }
+  }
+  return rounds - 1;
+}
+
 __device__ __forceinline__ uint32_t e4m3_byte(float v) { return e4m3x2(v, 0.f) & 0xFFu; }
 
 static_assert(kRQPartSmemBytes == kChunkPadded * 8 + 2 * kChunk + 16 * 8, "part scratch layout");
 
 // The share `part` of 16 / VPC parts of one row in the fused decode launch, for rows of
 // at most MAXCH chunks (K <= 4096 MAXCH; VPC * MAXCH <= 16): the codes and scale of
-// rotate_quant_row<kRQAct>, computed for low latency rather than throughput.
+// rotate_quant_row<kRQAct>, computed for low latency rather than throughput.  This code
+// runs once per launch, so its instructions are fetched cold; it is kept small (rolled
+// chunk loop, one butterfly body for all rounds) so that repeated work runs from the
+// instruction cache.
 //   * The next chunk's 32 bytes per thread are requested before the current chunk's
 //     butterflies run, so the row's global loads overlap the arithmetic.
 //   * The VPC values of each chunk that this part quantizes are converted to fp32 as the
@@ -654,67 +717,74 @@ __device__ __forceinline__ void rotate_quant_row_part_fast(const RQArgs& a, int 
     if (part == 0 && tid == 0 && a.scales != nullptr) a.scales[row] = 0.f;
     return;
   }
-  if (tid == 0) DPTQ_TRACE_CLOCK(tr, 160 + 10);
+  if (tid == 0) DPTQ_TRACE_CLOCK(tr, 170);
   const uint4* src = reinterpret_cast<const uint4*>(a.x + (size_t)row * K);
   float kept[MAXCH][VPC];
-  int kept_L[MAXCH];
+  int kept_L = 0;   // layout of every chunk (the same for all chunks of a row but a shorter last one)
+  int last_L = 0;
   long long mB = 0, mT = 0;
   uint4 u[2];
   rq_load16(src, 0, min(kChunk, K), tid, u);
+#pragma unroll 1
+  for (int c = 0; c < nch; ++c) {
+    const int c0 = c * kChunk;
+    const int len = min(kChunk, K - c0);
+    long long f[16];
+    rq_fix16(a, u, c0, len, tid, f);
+    if (c + 1 < nch) rq_load16(src, c0 + kChunk, min(kChunk, K - c0 - kChunk), tid, u);
+    if (tid == 0 && c == 0) DPTQ_TRACE_CLOCK(tr, 171);
+    const int L = rq_bfly_compact(a, c0, len, tail_start, f, sx, tid, sync);
+    if (tid == 0 && c == 0) DPTQ_TRACE_CLOCK(tr, 176);
+    if (c == 0) kept_L = L;
+    last_L = L;
+    if (len == kChunk && c0 + len <= tail_start) {   // every value is in a block of size B
 #pragma unroll
-  for (int c = 0; c < MAXCH; ++c) {
-    kept_L[c] = 0;
-    if (c < nch) {
-      const int c0 = c * kChunk;
-      const int len = min(kChunk, K - c0);
-      long long f[16];
-      rq_fix16(a, u, c0, len, tid, f);
-      if (c + 1 < nch) rq_load16(src, c0 + kChunk, min(kChunk, K - c0 - kChunk), tid, u);
-      const int L = rq_bfly(a, c0, len, tail_start, f, sx, tid, sync);
-      kept_L[c] = L;
-      if (len == kChunk && c0 + len <= tail_start) {   // every value is in a block of size B
-#pragma unroll
-        for (int e = 0; e < 16; ++e) {
-          const long long v = f[e] < 0 ? -f[e] : f[e];
-          mB = v > mB ? v : mB;
-        }
-      } else {
-#pragma unroll
-        for (int e = 0; e < 16; ++e) {
-          const int i = rq_pos(L, tid, e);
-          const long long v = f[e] < 0 ? -f[e] : f[e];
-          if (i < len) {
-            if (c0 + i < tail_start)
-              mB = v > mB ? v : mB;
-            else
-              mT = v > mT ? v : mT;
-          }
-        }
+      for (int e = 0; e < 16; ++e) {
+        const long long v = f[e] < 0 ? -f[e] : f[e];
+        mB = v > mB ? v : mB;
       }
-      long long v[VPC];   // f[e0 .. e0 + VPC - 1]; `part` is uniform over the CTA
-      if constexpr (VPC == 4) {
-        switch (part) {
-          case 0: v[0] = f[0]; v[1] = f[1]; v[2] = f[2]; v[3] = f[3]; break;
-          case 1: v[0] = f[4]; v[1] = f[5]; v[2] = f[6]; v[3] = f[7]; break;
-          case 2: v[0] = f[8]; v[1] = f[9]; v[2] = f[10]; v[3] = f[11]; break;
-          default: v[0] = f[12]; v[1] = f[13]; v[2] = f[14]; v[3] = f[15]; break;
+    } else {
+#pragma unroll
+      for (int e = 0; e < 16; ++e) {
+        const int i = rq_pos(L, tid, e);
+        const long long v = f[e] < 0 ? -f[e] : f[e];
+        if (i < len) {
+          if (c0 + i < tail_start)
+            mB = v > mB ? v : mB;
+          else
+            mT = v > mT ? v : mT;
         }
-      } else {
-        if (part == 0) {
-#pragma unroll
-          for (int j = 0; j < 8; ++j) v[j] = f[j];
-        } else {
-#pragma unroll
-          for (int j = 0; j < 8; ++j) v[j] = f[8 + j];
-        }
-      }
-#pragma unroll
-      for (int j = 0; j < VPC; ++j) {
-        const int i = rq_pos(L, tid, e0 + j);
-        kept[c][j] = i < len ? fixed_to_rotated(v[j], (c0 + i < tail_start) ? a.log2B : a.log2T, a.c_hi, a.c_lo)
-                             : 0.f;
       }
     }
+    long long v[VPC];   // f[e0 .. e0 + VPC - 1]; `part` is uniform over the CTA
+    if constexpr (VPC == 4) {
+      switch (part) {
+        case 0: v[0] = f[0]; v[1] = f[1]; v[2] = f[2]; v[3] = f[3]; break;
+        case 1: v[0] = f[4]; v[1] = f[5]; v[2] = f[6]; v[3] = f[7]; break;
+        case 2: v[0] = f[8]; v[1] = f[9]; v[2] = f[10]; v[3] = f[11]; break;
+        default: v[0] = f[12]; v[1] = f[13]; v[2] = f[14]; v[3] = f[15]; break;
+      }
+    } else {
+      if (part == 0) {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) v[j] = f[j];
+      } else {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) v[j] = f[8 + j];
+      }
+    }
+    float kv[VPC];
+#pragma unroll
+    for (int j = 0; j < VPC; ++j) {
+      const int i = rq_pos(L, tid, e0 + j);
+      kv[j] = i < len ? fixed_to_rotated(v[j], (c0 + i < tail_start) ? a.log2B : a.log2T, a.c_hi, a.c_lo) : 0.f;
+    }
+#pragma unroll
+    for (int cc = 0; cc < MAXCH; ++cc)   // kept[c] = kv with static register indices
+      if (cc == c) {
+#pragma unroll
+        for (int j = 0; j < VPC; ++j) kept[cc][j] = kv[j];
+      }
   }
   if (tid == 0) DPTQ_TRACE_CLOCK(tr, 140);
   // Row absmax (see above); the barrier also ends every read of sx.
@@ -735,29 +805,34 @@ __device__ __forceinline__ void rotate_quant_row_part_fast(const RQArgs& a, int 
   if (tid == 0) DPTQ_TRACE_CLOCK(tr, 141);
 
   // Codes of this part, staged at their k (plane 0 at stg[k], plane 1 at stg[K_pad + k]).
+#pragma unroll 1
+  for (int c = 0; c < nch; ++c) {
+    const int c0 = c * kChunk;
+    const int len = min(kChunk, K - c0);
+    const int L = c + 1 < nch ? kept_L : last_L;
+    float kv[VPC];
 #pragma unroll
-  for (int c = 0; c < MAXCH; ++c) {
-    if (c < nch) {
-      const int c0 = c * kChunk;
-      const int len = min(kChunk, K - c0);
-      const int L = kept_L[c];
+    for (int cc = 0; cc < MAXCH; ++cc)
+      if (cc == c) {
 #pragma unroll
-      for (int g4 = 0; g4 < VPC / 4; ++g4) {
-        float y[4] = {kept[c][4 * g4], kept[c][4 * g4 + 1], kept[c][4 * g4 + 2], kept[c][4 * g4 + 3]};
-        float q[4] = {0.f, 0.f, 0.f, 0.f};
-        if (nz) quant_code4(y, s, rs, qminf, qmaxf, q);
+        for (int j = 0; j < VPC; ++j) kv[j] = kept[cc][j];
+      }
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const int i = rq_pos(L, tid, e0 + 4 * g4 + j);
-          if (i < len) {
-            if (bits == 4) {
-              stg[c0 + i] = (uint8_t)e4m3_byte(q[j]);
-            } else {
-              const float m = fabsf(q[j]);
-              const float h = __fmul_rn(floorf(__fmul_rn(m, 0.0625f)), 16.f);
-              stg[c0 + i] = (uint8_t)e4m3_byte(__fadd_rn(copysignf(h, q[j]), 0.0f));
-              stg[K_pad + c0 + i] = (uint8_t)e4m3_byte(__fadd_rn(copysignf(__fsub_rn(m, h), q[j]), 0.0f));
-            }
+    for (int g4 = 0; g4 < VPC / 4; ++g4) {
+      float y[4] = {kv[4 * g4], kv[4 * g4 + 1], kv[4 * g4 + 2], kv[4 * g4 + 3]};
+      float q[4] = {0.f, 0.f, 0.f, 0.f};
+      if (nz) quant_code4(y, s, rs, qminf, qmaxf, q);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int i = rq_pos(L, tid, e0 + 4 * g4 + j);
+        if (i < len) {
+          if (bits == 4) {
+            stg[c0 + i] = (uint8_t)e4m3_byte(q[j]);
+          } else {
+            const float m = fabsf(q[j]);
+            const float h = __fmul_rn(floorf(__fmul_rn(m, 0.0625f)), 16.f);
+            stg[c0 + i] = (uint8_t)e4m3_byte(__fadd_rn(copysignf(h, q[j]), 0.0f));
+            stg[K_pad + c0 + i] = (uint8_t)e4m3_byte(__fadd_rn(copysignf(__fsub_rn(m, h), q[j]), 0.0f));
           }
         }
       }
@@ -766,19 +841,16 @@ __device__ __forceinline__ void rotate_quant_row_part_fast(const RQArgs& a, int 
   if (tid == 0) DPTQ_TRACE_CLOCK(tr, 142);
   sync();
   // The words whose values this part owns: value index of element i in layout L.
-#pragma unroll
-  for (int c = 0; c < MAXCH; ++c) {
-    if (c < nch) {
-      const int c0 = c * kChunk;
-      const int len = min(kChunk, K - c0);
-      const int L = kept_L[c];
-      for (int w = tid; w < len / 4; w += kRQThreads) {
-        const int i = 4 * w;
-        const int ei = L == 2 ? i >> 8 : L == 1 ? (i >> 4) & 15 : i & 15;
-        if (ei >= e0 && ei < e0 + VPC)
-          store4(c0 + i, *reinterpret_cast<const uint32_t*>(stg + c0 + i),
-                 *reinterpret_cast<const uint32_t*>(stg + K_pad + c0 + i));
-      }
+  for (int c = 0; c < nch; ++c) {
+    const int c0 = c * kChunk;
+    const int len = min(kChunk, K - c0);
+    const int L = c + 1 < nch ? kept_L : last_L;
+    for (int w = tid; w < len / 4; w += kRQThreads) {
+      const int i = 4 * w;
+      const int ei = L == 2 ? i >> 8 : L == 1 ? (i >> 4) & 15 : i & 15;
+      if (ei >= e0 && ei < e0 + VPC)
+        store4(c0 + i, *reinterpret_cast<const uint32_t*>(stg + c0 + i),
+               *reinterpret_cast<const uint32_t*>(stg + K_pad + c0 + i));
     }
   }
   if (part == NP - 1)   // k in [K, K_pad): zero codes
