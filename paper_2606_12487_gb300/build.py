@@ -36,6 +36,9 @@ def nvcc() -> str:
 def _flags():
     return ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I", os.path.join(ROOT, "include"),
                    *(["-DDPTQ_TRACE"] if TRACE else []),
+                   *([f"-DDPTQ_TRACE_STAGES={int(os.environ['DPTQ_TRACE_STAGES'])}"]
+                     if TRACE and os.environ.get("DPTQ_TRACE_STAGES") else []),
+                   *(["-DDPTQ_TRACE_CLOCKS"] if TRACE and os.environ.get("DPTQ_TRACE_CLOCKS") == "1" else []),
                    "--ptxas-options=-v" if os.environ.get("DPTQ_PTXAS_V") else "-Xptxas=-O3"]
 
 

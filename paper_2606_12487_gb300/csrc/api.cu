@@ -169,6 +169,12 @@ dptq_status ensure_scratch(int dev, size_t act_bytes, size_t sa_count, cudaStrea
       if (err) cudaFree(err);
       return cuda_fail(e, "scratch allocation");
     }
+    // DPTQ_MAX_GRID=n caps the CTAs of a GEMM launch (tuning experiments; default: the
+    // device's SMs).
+    if (const char* v = std::getenv("DPTQ_MAX_GRID")) {
+      const int cap = std::atoi(v);
+      if (cap > 0 && cap < sms) sms = cap;
+    }
     sc.num_sms = sms;
     sc.ws = ws;
     sc.counters = counters;

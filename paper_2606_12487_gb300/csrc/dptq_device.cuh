@@ -20,10 +20,27 @@ __device__ __forceinline__ unsigned long long trace_now() {
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
   return t;
 }
+#ifdef DPTQ_TRACE_CLOCKS
+// Stamps in SM cycles (cheap); the entry stamp also records %globaltimer (slot 0) and the
+// cycle counter (slot 255) so that CTAs can be put on one time axis.
+#define DPTQ_TRACE_POINT(buf, slot) \
+  do {                              \
+    if (buf) (buf)[blockIdx.x * 256 + (slot)] = (unsigned long long)clock64(); \
+  } while (0)
+#define DPTQ_TRACE_ENTRY(buf)                                                        \
+  do {                                                                               \
+    if (buf) {                                                                       \
+      (buf)[blockIdx.x * 256 + 255] = (unsigned long long)clock64();                \
+      (buf)[blockIdx.x * 256] = ::dptq::trace_now();                                \
+    }                                                                                \
+  } while (0)
+#else
 #define DPTQ_TRACE_POINT(buf, slot) \
   do {                              \
     if (buf) (buf)[blockIdx.x * 256 + (slot)] = ::dptq::trace_now(); \
   } while (0)
+#define DPTQ_TRACE_ENTRY(buf) DPTQ_TRACE_POINT(buf, 0)
+#endif
 #define DPTQ_TRACE_VALUE(buf, slot, v) \
   do {                                 \
     if (buf) (buf)[blockIdx.x * 256 + (slot)] = (unsigned long long)(v); \
@@ -44,6 +61,9 @@ __device__ __forceinline__ unsigned long long trace_now() {
   do {                                 \
   } while (0)
 #define DPTQ_TRACE_BUF() nullptr
+#define DPTQ_TRACE_ENTRY(buf) \
+  do {                        \
+  } while (0)
 #endif
 
 // Device error codes written to the library's error word (host maps them to status).

@@ -21,13 +21,17 @@
 // D[n][m] lives in TMEM with lane = output channel and column = token.
 //
 // Warp roles of the persistent CTA (one per SM):
-//   warp 0      producer: bulk copies (TMA engine) of packed weight tiles and of the
-//               pre-swizzled E4M3 activation tiles into a `stages`-deep ring; a stage
-//               holds KPS k-blocks of 128
+//   warp 0      weight producer: bulk copies (TMA engine) of packed weight tiles into a
+//               `stages`-deep ring (a stage holds KPS k-blocks of 128), from the start
 //   warp 1      TMEM allocator + single-thread tcgen05.mma issuer
-//   warps 2-9   converters: packed int4 -> E4M3 in the 128-byte swizzle layout
-//   warps 10-13 epilogue: tcgen05.ld -> int32 -> scales -> fp16, or int32 atomics into
+//   warps 2-9   converters: packed int4 -> E4M3 (into tensor memory, or shared memory
+//               in the 128-byte swizzle layout); in a fused launch they first rotate and
+//               quantize the token rows
+//   warps 10-13 epilogue: tcgen05.ld -> int32 -> scales -> fp16, or partial sums into
 //               the split-tile scratch, the last contributor finishing the tile
+//   warp 14     activation producer: bulk copies of the pre-swizzled E4M3 activation
+//               tiles into the same ring, once the previous kernel (and, fused, the row
+//               quantization) is done
 // Work: whole tiles round-robin first (`dp_tiles`), then the remaining tiles' k-blocks
 // split evenly over the CTAs (stream-K), so every SM streams the same number of
 // weight bytes.
@@ -42,8 +46,14 @@
 namespace dptq {
 
 constexpr int kNumConvWarps = 8, kConvWarp0 = 2;
+#ifndef DPTQ_TRACE_STAGES
+#define DPTQ_TRACE_STAGES 16
+#endif
+// Trace builds record per-stage stamps for the first kTraceStages stages of each role.
+constexpr int kTraceStages = DPTQ_TRACE_STAGES;
 constexpr int kNumEpiWarps = 4, kEpiWarp0 = kConvWarp0 + kNumConvWarps;
-constexpr int kGemmThreads = 32 * (kEpiWarp0 + kNumEpiWarps);   // 448
+constexpr int kActWarp = kEpiWarp0 + kNumEpiWarps;               // activation producer
+constexpr int kGemmThreads = 32 * (kActWarp + 1);                // 480
 constexpr int kConvThreads = 32 * kNumConvWarps;
 constexpr int kConvBytes = 128 * 128;   // one weight tile widened to E4M3
 constexpr int kMaxStages = 8;
@@ -171,6 +181,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
   // widen the weights straight into tensor memory and feed the MMA's A operand from
   // there; other one-block stages widen into shared memory.
   constexpr bool kATmem = a_in_tmem(NT, KPS);
+  // Two-block stages with the widened weights in tensor memory: the converter warps form
+  // two groups of four (one warp per TMEM lane quarter) that take alternate stages, each
+  // warp widening both k-blocks of its quarter, so that two stages convert at once.
+  constexpr bool kAltConv = kATmem && KPS == 2;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int S = a.stages;
@@ -181,8 +195,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
   uint64_t* empty = bars + kMaxStages;       // slot s: MMA done with it
   uint64_t* afull = bars + 2 * kMaxStages;   // slot s: activation copies landed
   uint64_t* cfull = bars + 3 * kMaxStages;   // widened slot c: written
-  uint64_t* cempty = cfull + kMaxConvSlots;  // widened slot c: MMA done with it
-  uint64_t* tfull = cempty + kMaxConvSlots;
+  uint64_t* tfull = cfull + 2 * kMaxConvSlots;
   uint64_t* tempty = tfull + 2;
   uint64_t* drain = tempty + 2;
   uint64_t* esync = drain + 1;   // epilogue-group barrier (4 warps), bounded waits
@@ -193,13 +206,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
   float* sa_sh = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + 512);   // token scales (NT <= 64)
   __half* xpose = reinterpret_cast<__half*>(reinterpret_cast<uint8_t*>(bars) + 1024);  // 4 x [4 tokens][32 ch]
   unsigned char* rot_smem = reinterpret_cast<unsigned char*>(bars) + kBarrierBytes;    // fused: one row's scratch
-  const uint8_t** pend_src = reinterpret_cast<const uint8_t**>(tmem_base_sh + 8);   // producer's pending list
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   unsigned long long* const tr = DPTQ_TRACE_BUF();
   (void)tr;
-  if (threadIdx.x == 0) DPTQ_TRACE_POINT(tr, 0);
+  if (threadIdx.x == 0) DPTQ_TRACE_ENTRY(tr);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
@@ -208,8 +220,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
       mbar_init(&afull[s], 1);
     }
     for (int c = 0; c < CS; ++c) {
-      mbar_init(&cfull[c], kNumConvWarps);
-      mbar_init(&cempty[c], 1);
+      mbar_init(&cfull[c], kAltConv ? kNumConvWarps / 2 : kNumConvWarps);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&tfull[b], 1);
@@ -237,11 +248,18 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
   iter.init(a);
   Unit un;
 
-  if (warp == 0) {
-    // ------------------------------------------------------------ producer
-    // Whole warp, uniform control flow; the elected leader issues the copies.
+  if (warp == 0 || warp == kActWarp) {
+    // ------------------------------------------------------------ producers
+    // Warp 0 streams the packed weight tiles, which do not depend on the previous kernel,
+    // from the first moment; warp kActWarp requests the activation tiles, which do: it
+    // waits for the previous kernel (programmatic dependent launch) and, in a fused
+    // launch, for every token row to be published, then follows the ring.  Both walk the
+    // same stages and wait for the same `empty` barriers; each arms its own barrier of a
+    // stage (`full`: weights, `afull`: activations).  Whole warps, uniform control flow;
+    // an elected leader issues the copies.
+    const bool wprod = warp == 0;
     const bool leader = elect_one();
-    if (leader) DPTQ_TRACE_POINT(tr, 117);
+    if (leader && wprod) DPTQ_TRACE_POINT(tr, 117);
     const uint64_t pol_w = l2_policy_evict_first();   // weights are streamed once
     const uint64_t pol_a = l2_policy_evict_last();    // activations are re-read per n-tile
     const uint32_t act_bytes = (uint32_t)NT * 128;
@@ -249,54 +267,14 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
     const uint32_t a_tx = (uint32_t)(KPS * a.planes) * act_bytes;
     const size_t plane_stride = (size_t)a.KB * a.M_pad * 128;
     const size_t kb_stride = (size_t)a.M_pad * 128;
-    auto issue_act = [&](int slot, const uint8_t* src) {
-      mbar_arrive_expect_tx(&afull[slot], a_tx);
-#pragma unroll
-      for (int h = 0; h < KPS; ++h)
-        for (int pl = 0; pl < a.planes; ++pl)
-          bulk_g2s(sm.act(slot, h, pl), src + h * kb_stride + pl * plane_stride, act_bytes, &afull[slot], pol_a);
-    };
-    // Activation tiles may be requested once the previous kernel has finished
-    // (programmatic dependent launch) and, in a fused launch, every token row has been
-    // quantized.  False only when the CTA aborts.
-    auto act_ready = [&]() -> bool {
-      pdl_wait();
-      if constexpr (FUSED) {
-        const long long t0 = clock64();
-        while (true) {
-          int st = 0;
-          if (lane == 0) {
-            if (ld_acquire_gpu(a.gsync) >= (uint32_t)a.rq_items)
-              st = 1;
-            else if (*abort_flag)
-              st = 2;
-            else if (clock64() - t0 > kWaitTimeoutCycles) {
-              *abort_flag = 1;
-              atomicCAS(a.err, 0, (int)kDevTimeoutGrid);
-              st = 2;
-            }
-          }
-          st = __shfl_sync(0xffffffffu, st, 0);
-          if (st == 1) break;
-          if (st == 2) return false;
-          __nanosleep(32);
-        }
-        fence_proxy_async_global();   // the bulk copies read what other CTAs stored
-        if (leader) {
-          DPTQ_TRACE_POINT(tr, 116);
-          mbar_arrive(aready);
-        }
-      }
-      return true;
-    };
-    // Decode launches: once the first S stages are requested, the rest of this CTA's
-    // weight share (up to a cap) is requested into L2 in one go, so that HBM streams the
-    // weights while the token rows are rotated and published, instead of only as fast as
-    // the ring frees stages.  Units are visited in processing order; each unit's weight
-    // range is contiguous (tile-major, k-blocks consecutive) and, with one token tile,
-    // belongs to this CTA alone.
+    // Decode launches: once the ring's first S stages are requested, the weight producer
+    // requests the rest of its CTA's share (up to a cap) into L2, so that HBM streams the
+    // weights while the ring is still full (the token rows are being rotated, or the
+    // previous kernel finishes).  Units are visited in processing order; each unit's
+    // weight range is contiguous (tile-major, k-blocks consecutive) and, with one token
+    // tile, belongs to this CTA.
     auto prefetch_share = [&]() {
-      if (a.l2_prefetch <= 0 || !leader) return;
+      if (!(wprod && leader && a.l2_prefetch > 0)) return;
       UnitIter pit;
       pit.init(a);
       Unit pu;
@@ -319,70 +297,87 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
           bulk_prefetch_l2(base + off, (uint32_t)(len - off < 32768 ? len - off : 32768));
       }
     };
-    // Weight tiles do not depend on the previous kernel; the first `S` stages are
-    // requested before waiting for it and their activation halves are issued once
-    // act_ready() returns (also after an abort, so that every armed stage completes).
-    bool waited = false;
-    int npend = 0;
+    // The activation producer starts once the previous kernel has finished and, in a fused
+    // launch, every token row has been quantized.
+    bool ok = true;
+    if (!wprod) {
+      pdl_wait();
+      if constexpr (FUSED) {
+        const long long t0 = clock64();
+        while (true) {
+          int st = 0;
+          if (lane == 0) {
+            if (ld_acquire_gpu(a.gsync) >= (uint32_t)a.rq_items)
+              st = 1;
+            else if (*abort_flag)
+              st = 2;
+            else if (clock64() - t0 > kWaitTimeoutCycles) {
+              *abort_flag = 1;
+              atomicCAS(a.err, 0, (int)kDevTimeoutGrid);
+              st = 2;
+            }
+          }
+          st = __shfl_sync(0xffffffffu, st, 0);
+          if (st == 1) break;
+          if (st == 2) {
+            ok = false;
+            break;
+          }
+          __nanosleep(32);
+        }
+        if (ok) {
+          fence_proxy_async_global();   // the bulk copies read what other CTAs stored
+          if (leader) {
+            DPTQ_TRACE_POINT(tr, 116);
+            mbar_arrive(aready);
+          }
+        }
+      }
+    }
     Ring rg(S);
     int g = 0;
-    bool ok = true;
     while (ok && iter.next(un)) {
       const int nt = un.tile / a.m_tiles;
       const int mt = un.tile - nt * a.m_tiles;
-      if (leader) DPTQ_TRACE_POINT(tr, 118);
+      if (leader && wprod) DPTQ_TRACE_POINT(tr, 118);
       const uint8_t* wsrc = a.wt + ((size_t)nt * a.KB + (size_t)un.i0 * KPS) * kWTileBytes;
       const uint8_t* asrc = a.act + ((size_t)un.i0 * KPS * a.M_pad + (size_t)mt * NT) * 128;
       for (int it = un.i0; it < un.i1; ++it, ++g, rg.next(), wsrc += w_bytes, asrc += KPS * kb_stride) {
         const int s = rg.s;
-        if (leader && g == 8) DPTQ_TRACE_CLOCK(tr, 242);
+        const bool tg = kTraceStages > 10 && wprod && leader && g >= 8 && g < 11;   // clocked stages (trace builds)
+        (void)tg;
+        if (tg) DPTQ_TRACE_CLOCK(tr, 224 + 3 * (g - 8));
         if (!mbar_wait_warp(&empty[s], rg.ph ^ 1u, abort_flag, a.err, kDevTimeoutEmpty)) {
           ok = false;
           break;
         }
         if (leader) {
-          if (g == 8) DPTQ_TRACE_CLOCK(tr, 241);
-          if (g < 16) DPTQ_TRACE_POINT(tr, 8 + g);
-          mbar_arrive_expect_tx(&full[s], w_bytes);
-          bulk_g2s(sm.wpack(s), wsrc, w_bytes, &full[s], pol_w);
-          if (waited)
-            issue_act(s, asrc);
-          else
-            pend_src[npend] = asrc;   // stage index of pending entry i is i
-          if (g < 16) DPTQ_TRACE_POINT(tr, 24 + g);
-        }
-        if (!waited && ++npend == S) {
-          prefetch_share();
-          if (!act_ready()) ok = false;
-          waited = true;
-          __syncwarp();
-          if (leader)
-            for (int i = 0; i < npend; ++i) issue_act(i, pend_src[i]);
-          npend = 0;
+          if (tg) DPTQ_TRACE_CLOCK(tr, 225 + 3 * (g - 8));
+          if (wprod) {
+            if (g < kTraceStages) DPTQ_TRACE_POINT(tr, 8 + g);
+            mbar_arrive_expect_tx(&full[s], w_bytes);
+            bulk_g2s(sm.wpack(s), wsrc, w_bytes, &full[s], pol_w);
+            if (g < kTraceStages) DPTQ_TRACE_POINT(tr, 24 + g);
+            if (g == S - 1) prefetch_share();
+          } else {
+            mbar_arrive_expect_tx(&afull[s], a_tx);
+#pragma unroll
+            for (int h = 0; h < KPS; ++h)
+              for (int pl = 0; pl < a.planes; ++pl)
+                bulk_g2s(sm.act(s, h, pl), asrc + h * kb_stride + pl * plane_stride, act_bytes, &afull[s], pol_a);
+          }
+          if (tg) DPTQ_TRACE_CLOCK(tr, 226 + 3 * (g - 8));
         }
         __syncwarp();
-        if (!ok) {
-          ++g;   // this stage is armed: the drain below must see it
-          break;
-        }
       }
-    }
-    // Stages armed before the wait for the previous kernel still expect their
-    // activation bytes (also after an abort, so that the drain below completes).
-    if (!waited) {
-      act_ready();
-      __syncwarp();
-      if (leader)
-        for (int i = 0; i < npend; ++i) issue_act(i, pend_src[i]);
     }
     __syncwarp();
-    // Do not leave the CTA while copies into its shared memory may be in flight.
+    // Do not leave the CTA while copies into its shared memory may be in flight: after an
+    // abort, wait (bounded) for the copies this warp armed in the last S stages.
     if (*abort_flag) {
       volatile int no_abort = 0;
-      for (int gg = (g > S ? g - S : 0); gg < g; ++gg) {
-        mbar_wait_warp(&full[gg % S], (gg / S) & 1, &no_abort, a.err, kDevTimeoutDrain);
-        mbar_wait_warp(&afull[gg % S], (gg / S) & 1, &no_abort, a.err, kDevTimeoutDrain);
-      }
+      for (int gg = (g > S ? g - S : 0); gg < g; ++gg)
+        mbar_wait_warp(wprod ? &full[gg % S] : &afull[gg % S], (gg / S) & 1, &no_abort, a.err, kDevTimeoutDrain);
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
@@ -414,19 +409,21 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
       bool ok = true;
       for (int it = un.i0; it < un.i1; ++it, rg.next(), rc.next()) {
         const int s = rg.s, c = rc.s;
-        if (leader && it - un.i0 + mma_done == 8) DPTQ_TRACE_CLOCK(tr, 237);
+        const int gm = it - un.i0 + mma_done;
+        const bool tgm = kTraceStages > 10 && leader && gm >= 8 && gm < 11;   // stages whose steps are clocked (trace builds)
+        (void)tgm;
+        if (tgm) DPTQ_TRACE_CLOCK(tr, 200 + 8 * (gm - 8));
         if (!mbar_wait_warp(&afull[s], rg.ph, abort_flag, a.err, kDevTimeoutFull)) {
           ok = false;
           break;
         }
-        if (leader && it - un.i0 + mma_done == 8) DPTQ_TRACE_CLOCK(tr, 239);
+        if (tgm) DPTQ_TRACE_CLOCK(tr, 201 + 8 * (gm - 8));
         if (!mbar_wait_warp(&cfull[c], rc.ph, abort_flag, a.err, kDevTimeoutConv)) {
           ok = false;
           break;
         }
-        const int gm = it - un.i0 + mma_done;
-        if (leader && gm == 8) DPTQ_TRACE_CLOCK(tr, 235);
-        if (leader && gm < 16) DPTQ_TRACE_POINT(tr, 72 + gm);
+        if (tgm) DPTQ_TRACE_CLOCK(tr, 202 + 8 * (gm - 8));
+        if (leader && gm < kTraceStages) DPTQ_TRACE_POINT(tr, 72 + gm);
         tc_fence_after();
         if (seg_left == 0) {   // next exact-accumulation segment: next accumulator
           d += NT;
@@ -454,12 +451,16 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
               }
             }
           }
+          if (tgm) DPTQ_TRACE_CLOCK(tr, 203 + 8 * (gm - 8));
+          // One commit per stage: it frees the bulk-copy slot (producer) and tells the
+          // converters that widened slot c may be overwritten (they wait on the same
+          // barrier, one ring position CS stages back).
           mma_commit(&empty[s]);
-          mma_commit(&cempty[c]);
-          if (gm == 8) DPTQ_TRACE_CLOCK(tr, 236);
-          if (gm < 16) DPTQ_TRACE_POINT(tr, 88 + gm);
+          if (tgm) DPTQ_TRACE_CLOCK(tr, 205 + 8 * (gm - 8));
+          if (gm < kTraceStages) DPTQ_TRACE_POINT(tr, 88 + gm);
         }
         __syncwarp();
+        if (tgm) DPTQ_TRACE_CLOCK(tr, 206 + 8 * (gm - 8));
         fresh = 0;
         --seg_left;
       }
@@ -469,6 +470,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
       mma_done += un.i1 - un.i0;
       ++u;
     }
+    if (leader) DPTQ_TRACE_POINT(tr, 124);   // last MMA issued
     // Every MMA the leader issued must be complete before TMEM is released.
     if (leader) mma_commit(drain);
     __syncwarp();
@@ -506,26 +508,78 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
       }
       if (ctid == 0) DPTQ_TRACE_POINT(tr, 127);
     }
-    Ring rg(S), rc(CS);
-    int cvt_done = 0;
+    // rl trails rg by CS stages: the MMA of stage gc - CS was the last to read widened
+    // slot c, and its commit completes that stage's `empty` barrier.
+    Ring rg(S), rc(CS), rl(S);
+    const int grp = (warp - kConvWarp0) >> 2;   // converter group (alternate stages)
+    const int tid_grp = (warp - kConvWarp0 - 4 * grp) * 32 + lane;
+    (void)tid_grp;
+    int gc = 0;
     while (iter.next(un)) {
       bool ok = true;
-      for (int it = un.i0; it < un.i1; ++it, rg.next(), rc.next()) {
+      for (int it = un.i0; it < un.i1; ++it, ++gc, rg.next(), rc.next()) {
         const int s = rg.s, c = rc.s;
-        if (ctid == 0 && it - un.i0 + cvt_done == 8) DPTQ_TRACE_CLOCK(tr, 238);
+        if (gc > CS) rl.next();   // rl = ring position of stage gc - CS (from gc = CS on)
+        if (kAltConv && (gc & 1) != grp) continue;   // the other group's stage
+        const bool tgc = kTraceStages > 10 && (kAltConv ? tid_grp == 0 : ctid == 0) && gc >= 8 && gc < 11;   // clocked (trace builds)
+        (void)tgc;
+        if (tgc) DPTQ_TRACE_CLOCK(tr, 180 + 6 * (gc - 8));
+        // First the MMA of stage gc - CS (widened slot c free).  It also orders the wait
+        // on full[s]: a parity wait cannot tell a phase from the one two phases later,
+        // and a group that skips stages could otherwise look at slot s while its previous
+        // copy (stage gc - S, converted by the other group) is still in flight.  With
+        // S >= CS, that copy has landed and been consumed once the MMA of stage gc - CS
+        // is done.
+        if (gc >= CS && !mbar_wait(&empty[rl.s], rl.ph, abort_flag, a.err, kDevTimeoutConv)) {
+          ok = false;
+          break;
+        }
+        if (tgc) DPTQ_TRACE_CLOCK(tr, 181 + 6 * (gc - 8));
         if (!mbar_wait(&full[s], rg.ph, abort_flag, a.err, kDevTimeoutFull)) {
           ok = false;
           break;
         }
-        if (ctid == 0 && it - un.i0 + cvt_done == 8) DPTQ_TRACE_CLOCK(tr, 240);
-        if (!mbar_wait(&cempty[c], rc.ph ^ 1u, abort_flag, a.err, kDevTimeoutConv)) {
-          ok = false;
-          break;
-        }
-        const int gc = it - un.i0 + cvt_done;
-        if (ctid == 0 && gc < 16) DPTQ_TRACE_POINT(tr, 40 + gc);
+        if (tgc) DPTQ_TRACE_CLOCK(tr, 182 + 6 * (gc - 8));
+        if ((kAltConv ? tid_grp == 0 : ctid == 0) && gc < kTraceStages) DPTQ_TRACE_POINT(tr, 40 + gc);
         const uint8_t* __restrict__ wp = sm.wpack(s);
-        if constexpr (kATmem && KPS == 1) {
+        if constexpr (kAltConv) {
+          // Warp of lane quarter q widens both k-blocks of rows 32q..32q+31: each thread
+          // reads its row's 2 x 64 packed bytes (4 chunks of 32 k per block) and stores
+          // 2 x 32 columns of its TMEM lane.
+          tc_fence_after();
+          const int q = warp & 3;
+          const uint8_t* src = wp + (q * 32 + lane) * 16;
+          uint4 w[8];
+#pragma unroll
+          for (int j = 0; j < 8; ++j) w[j] = *reinterpret_cast<const uint4*>(src + (j >> 2) * kWTileBytes + (j & 3) * 2048);
+#ifdef DPTQ_TRACE
+          if (tgc) {
+            volatile uint32_t sink = w[0].x ^ w[7].w;
+            (void)sink;
+            DPTQ_TRACE_CLOCK(tr, 183 + 6 * (gc - 8));
+          }
+#endif
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            uint32_t v[32];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+              const uint4 ww = w[4 * h + j];
+              v[8 * j + 0] = widen_lo(ww.x);
+              v[8 * j + 1] = widen_hi(ww.x);
+              v[8 * j + 2] = widen_lo(ww.y);
+              v[8 * j + 3] = widen_hi(ww.y);
+              v[8 * j + 4] = widen_lo(ww.z);
+              v[8 * j + 5] = widen_hi(ww.z);
+              v[8 * j + 6] = widen_lo(ww.w);
+              v[8 * j + 7] = widen_hi(ww.w);
+            }
+            tmem_st32(tmem_base + ((uint32_t)(q * 32) << 16) + a.a_col0 + (uint32_t)((c * KPS + h) * 32), v);
+          }
+          tmem_st_wait();
+          tc_fence_before();
+          if (tgc) DPTQ_TRACE_CLOCK(tr, 184 + 6 * (gc - 8));
+        } else if constexpr (kATmem && KPS == 1) {
           // Warp (lane quarter q, half hs) widens k columns 64 hs .. 64 hs + 63 of rows
           // 32q..32q+31: each thread reads its row's 32 packed bytes (chunks 2 hs and
           // 2 hs + 1 of 32 k) and stores 16 columns of its TMEM lane.
@@ -549,32 +603,6 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
             v[8 * j + 7] = widen_hi(w[j].w);
           }
           tmem_st16(tmem_base + ((uint32_t)(q * 32) << 16) + a.a_col0 + (uint32_t)(c * 32 + hs * 16), v);
-          tmem_st_wait();
-          tc_fence_before();
-        } else if constexpr (kATmem) {
-          // Warp (lane quarter q, half hs) widens k-block hs of rows 32q..32q+31: each
-          // thread reads its row's 64 packed bytes (4 chunks of 32 k) and stores 32 columns
-          // of its TMEM lane.
-          tc_fence_after();
-          const int q = warp & 3;
-          const int hs = (warp - kConvWarp0) >> 2;
-          const uint8_t* src = wp + hs * kWTileBytes + (q * 32 + lane) * 16;
-          uint4 w[4];
-#pragma unroll
-          for (int j = 0; j < 4; ++j) w[j] = *reinterpret_cast<const uint4*>(src + j * 2048);
-          uint32_t v[32];
-#pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            v[8 * j + 0] = widen_lo(w[j].x);
-            v[8 * j + 1] = widen_hi(w[j].x);
-            v[8 * j + 2] = widen_lo(w[j].y);
-            v[8 * j + 3] = widen_hi(w[j].y);
-            v[8 * j + 4] = widen_lo(w[j].z);
-            v[8 * j + 5] = widen_hi(w[j].z);
-            v[8 * j + 6] = widen_lo(w[j].w);
-            v[8 * j + 7] = widen_hi(w[j].w);
-          }
-          tmem_st32(tmem_base + ((uint32_t)(q * 32) << 16) + a.a_col0 + (uint32_t)((c * KPS + hs) * 32), v);
           tmem_st_wait();
           tc_fence_before();
         } else {
@@ -613,11 +641,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(&cfull[c]);
-        if (ctid == 0 && gc == 8) DPTQ_TRACE_CLOCK(tr, 234);
-        if (ctid == 0 && gc < 16) DPTQ_TRACE_POINT(tr, 56 + gc);
+        if (tgc) DPTQ_TRACE_CLOCK(tr, 185 + 6 * (gc - 8));
+        if ((kAltConv ? tid_grp == 0 : ctid == 0) && gc < kTraceStages) DPTQ_TRACE_POINT(tr, 56 + gc);
       }
       if (!ok) break;
-      cvt_done += un.i1 - un.i0;
     }
   } else {
     // ------------------------------------------------------------ epilogue
@@ -970,6 +997,10 @@ bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan, i
   int stages = kMaxStages;
   while (stages > 2 && smem_total(stages) > kSmemLimit) --stages;
   if (smem_total(stages) > kSmemLimit || (fused && stages < 3)) return false;
+  // The converters learn that a widened slot is free from the `empty` barrier of the
+  // stage that last read it, CS stages back; with CS <= stages that barrier cannot
+  // complete a further phase before they look.
+  if (conv_slots > stages) conv_slots = stages;
   const int a_cols = a_tmem ? conv_slots * kps * 32 : 0;
   const int nbuf = 2 * nt * segs + a_cols <= 512 ? 2 : 1;
   if (nbuf * nt * segs + a_cols > 512) return false;
@@ -985,6 +1016,18 @@ bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan, i
   const long long iters = tiles * KI;
   int G = (int)(iters < num_sms ? iters : num_sms);
   if (G < 1) G = 1;
+  if (nt <= 64 && m_tiles == 1) {
+    // Decode (one token tile, weights streamed once).  A tile split over several CTAs costs
+    // its contributors fp32 reductions through L2 and a fence, and the tile's finisher an
+    // extra round trip at the end of the launch; measured on GB300 that outweighs a
+    // longer stream per CTA.  So: whole tiles, one per CTA, when they fit on the SMs and a
+    // tile is at most twice a CTA's fair share of the stages; otherwise stream-K with at
+    // most four CTAs per tile.
+    if (tiles <= num_sms && (long long)KI * num_sms <= 2 * iters)
+      G = (int)tiles;
+    else if (4 * tiles < G)
+      G = (int)(4 * tiles);
+  }
   long long dp = 0;
   if (tiles >= 2LL * G) dp = (tiles / G - 1) * G;
 

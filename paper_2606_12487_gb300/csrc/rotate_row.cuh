@@ -615,15 +615,26 @@ __device__ __forceinline__ int rq_bfly_compact(const RQArgs& a, int c0, int len,
   // Blocks are B-sized before tail_start and tail-sized after, so only chunks that reach
   // the tail can mix block sizes.
   const bool mixed = c0 + len > tail_start && a.log2T != a.log2B;
+  // Padded index of value e of this thread in layout r: pad_idx(rq_pos(r, tid, e)) =
+  // pb[r] + ps[r] e, since every layout is linear in e (strides 1, 16, 256) and the
+  // padding adds one slot per 16 elements.
+  const int pb0 = 17 * tid;
+  const int ib1 = 256 * (tid >> 4) + (tid & 15);
+  const int pb1 = ib1 + (ib1 >> 4);
+  const int pb2 = tid + (tid >> 4);
 #pragma unroll 1
   for (int r = 0; r < rounds; ++r) {
     if (r > 0) {
+      const int wb = r == 1 ? pb0 : pb1, ws = r == 1 ? 1 : 17;
+      const int rb = r == 1 ? pb1 : pb2, rs = r == 1 ? 17 : 272;
       sync();   // the previous readers of sx are done
+      long long* wp = sx + wb;
 #pragma unroll
-      for (int e = 0; e < 16; ++e) sx[pad_idx(rq_pos(r - 1, tid, e))] = f[e];
+      for (int e = 0; e < 16; ++e) wp[ws * e] = f[e];
       sync();
+      const long long* rp = sx + rb;
 #pragma unroll
-      for (int e = 0; e < 16; ++e) f[e] = sx[pad_idx(rq_pos(r, tid, e))];
+      for (int e = 0; e < 16; ++e) f[e] = rp[rs * e];
     }
     const int base = 4 * r;
     if (!mixed && a.log2B >= base + 4) {   // every element's block spans the round's 4 levels
