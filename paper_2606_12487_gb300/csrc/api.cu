@@ -261,6 +261,14 @@ bool l2_prefetch_allowed() {
   return on;
 }
 
+bool rows_kernel_allowed() {
+  static const bool on = [] {
+    const char* v = std::getenv("DPTQ_ROWS_KERNEL");
+    return !(v && v[0] == '0');
+  }();
+  return on;
+}
+
 // Record the message returned by dptq_last_error_message for this thread.
 void set_error_message(const std::string& m) { g_msg = m; }
 }  // namespace dptq

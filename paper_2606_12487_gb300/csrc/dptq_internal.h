@@ -154,6 +154,10 @@ bool pdl_allowed();
 bool fused_allowed();
 // Decode GEMM launches prefetch their weight share into L2 unless DPTQ_L2PF=0.
 bool l2_prefetch_allowed();
+// The GEMM operand rows are rotated and quantized by the whole-row kernel (sums kept in
+// registers) unless DPTQ_ROWS_KERNEL=0 (the per-row kernel with an fp32 row in shared
+// memory).
+bool rows_kernel_allowed();
 
 // The fixed scratch of dptq_qlinear_static on device `dev`: read its device error word
 // into *word and, when it is non-zero, clear the word, the split-tile sums and the

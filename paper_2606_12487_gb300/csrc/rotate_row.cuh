@@ -749,11 +749,17 @@ __device__ __forceinline__ void rotate_quant_row_part_fast(const RQArgs& a, int 
     if (c == 0) kept_L = L;
     last_L = L;
     if (len == kChunk && c0 + len <= tail_start) {   // every value is in a block of size B
+      long long m[8];   // pairwise tree: four dependent steps instead of sixteen
 #pragma unroll
-      for (int e = 0; e < 16; ++e) {
-        const long long v = f[e] < 0 ? -f[e] : f[e];
-        mB = v > mB ? v : mB;
+      for (int e = 0; e < 8; ++e) {
+        const long long p = f[e] < 0 ? -f[e] : f[e], q = f[e + 8] < 0 ? -f[e + 8] : f[e + 8];
+        m[e] = p > q ? p : q;
       }
+#pragma unroll
+      for (int w = 4; w > 0; w >>= 1)
+#pragma unroll
+        for (int e = 0; e < w; ++e) m[e] = m[e] > m[e + w] ? m[e] : m[e + w];
+      mB = m[0] > mB ? m[0] : mB;
     } else {
 #pragma unroll
       for (int e = 0; e < 16; ++e) {
@@ -851,15 +857,25 @@ __device__ __forceinline__ void rotate_quant_row_part_fast(const RQArgs& a, int 
   }
   if (tid == 0) DPTQ_TRACE_CLOCK(tr, 142);
   sync();
-  // The words whose values this part owns: value index of element i in layout L.
+  // The words whose values this part owns, VPC / 4 per thread and chunk, found directly
+  // from the layout: L = 2: k = 256 e + t, the part's values fill [256 e0, 256 (e0 + VPC));
+  // L = 1: k = 256 (t >> 4) + 16 e + (t & 15), the part's values fill 16 e0 .. 16 (e0 + VPC)
+  // within every 256-element block; L = 0: k = 16 t + e, the part's values are
+  // 16 t + e0 .. 16 t + e0 + VPC.
   for (int c = 0; c < nch; ++c) {
     const int c0 = c * kChunk;
     const int len = min(kChunk, K - c0);
     const int L = c + 1 < nch ? kept_L : last_L;
-    for (int w = tid; w < len / 4; w += kRQThreads) {
-      const int i = 4 * w;
-      const int ei = L == 2 ? i >> 8 : L == 1 ? (i >> 4) & 15 : i & 15;
-      if (ei >= e0 && ei < e0 + VPC)
+#pragma unroll
+    for (int j = 0; j < VPC / 4; ++j) {
+      int i;
+      if (L == 2)
+        i = 256 * e0 + 4 * (j * kRQThreads + tid);
+      else if (L == 1)
+        i = 256 * (tid >> 4) + 16 * e0 + 4 * (j * 16 + (tid & 15));
+      else
+        i = 16 * tid + e0 + 4 * j;
+      if (i < len)
         store4(c0 + i, *reinterpret_cast<const uint32_t*>(stg + c0 + i),
                *reinterpret_cast<const uint32_t*>(stg + K_pad + c0 + i));
     }
