@@ -49,6 +49,12 @@ def _load():
             lib.orc_float_to_half.restype = ctypes.c_uint16
             lib.orc_hadamard_entry.argtypes = [I, I]
             lib.orc_hadamard_entry.restype = I
+            lib.orc_paley_entry.argtypes = [I, I, I]
+            lib.orc_paley_entry.restype = I
+            lib.orc_tail_factor.argtypes = [I, P, P]
+            lib.orc_tail_factor.restype = I
+            lib.orc_tail_entry.argtypes = [I, I, I]
+            lib.orc_tail_entry.restype = I
             lib.orc_block_layout.argtypes = [I, I, P, P]
             lib.orc_block_layout.restype = I
             lib.orc_rotate_row_f64.argtypes = [P, P, I, I]
@@ -113,6 +119,24 @@ def float_to_half(v: float) -> int:
 
 def hadamard_entry(i: int, j: int) -> int:
     return int(_load().orc_hadamard_entry(i, j))
+
+
+def paley_entry(p: int, i: int, j: int) -> int:
+    """Entry of Paley's type-I Hadamard matrix of order p (p - 1 prime, = 3 mod 4); 0 when
+    p is not such an order."""
+    return int(_load().orc_paley_entry(p, i, j))
+
+
+def tail_factor(r: int):
+    """(p, k) with r = p 2^k for a tail block (p = 1 for a power of two), or None."""
+    p = ctypes.c_int(0)
+    k = ctypes.c_int(0)
+    return (p.value, k.value) if _load().orc_tail_factor(r, ctypes.byref(p), ctypes.byref(k)) else None
+
+
+def tail_entry(r: int, i: int, j: int) -> int:
+    """Entry (i, j) of the tail block's Hadamard matrix H_p (x) H_(2^k) of order r."""
+    return int(_load().orc_tail_entry(r, i, j))
 
 
 def block_layout(K: int, B: int):

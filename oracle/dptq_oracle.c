@@ -26,7 +26,8 @@
  *   - all-zero row: s = 0, every code 0;
  *   - R = blockdiag(H_B, ..., H_B, H_r) / sqrt(block), H the Sylvester Hadamard
  *     matrix in natural order, H[i][j] = (-1)^popcount(i & j); the tail block r is
- *     what is left of K after whole blocks of B (a power of two);
+ *     what is left of K after whole blocks of B: a power of two, or p 2^k with H_r the
+ *     Kronecker product of Paley's H_p and the Sylvester H_(2^k) (orc_tail_factor);
  *   - scales in fp32; epilogue out = fp16_rne( fp32( fp32(acc) * s_a ) * s_w ).
  *
  * Precision: the rotation is evaluated in fp64 and rounded once to fp32.  For fp16
@@ -110,18 +111,93 @@ int orc_hadamard_entry(int i, int j) {
 
 static int is_pow2(int v) { return v > 0 && (v & (v - 1)) == 0; }
 
+static int is_prime(long v) {
+    if (v < 2) return 0;
+    for (long d = 2; d * d <= v; ++d)
+        if (v % d == 0) return 0;
+    return 1;
+}
+
+/* Quadratic character of a modulo the odd prime q: 0 for a = 0 (mod q), +1 for a
+ * non-zero square, -1 otherwise (Euler's criterion, a^((q-1)/2) mod q). */
+static int legendre(long a, long q) {
+    long x = ((a % q) + q) % q;
+    if (x == 0) return 0;
+    long e = (q - 1) / 2, r = 1, b = x;
+    while (e) {
+        if (e & 1) r = (r * b) % q;
+        b = (b * b) % q;
+        e >>= 1;
+    }
+    return r == 1 ? 1 : -1;
+}
+
+/* Paley's first construction: for a prime q = p - 1 with q = 3 (mod 4),
+ * H_p = I + S with S[0][0] = 0, S[0][j] = +1, S[i][0] = -1 and S[i][j] = chi(j - i)
+ * (the Jacobsthal matrix of the quadratic character chi mod q) for i, j >= 1.  Because
+ * chi(-1) = -1, S is skew-symmetric and H_p H_p^T = p I.  Entry (i, j), 0 <= i, j < p;
+ * 0 when p is not such an order. */
+int orc_paley_entry(int p, int i, int j) {
+    if (p < 4 || p % 4 != 0 || !is_prime(p - 1)) return 0;
+    if (i == j) return 1;
+    if (i == 0) return 1;
+    if (j == 0) return -1;
+    return legendre((long)j - (long)i, p - 1);
+}
+
+/* Reading of the rotation for a tail block whose size r is not a power of two: the
+ * Kronecker product H_p (x) H_(2^k) with r = p 2^k, H_p from Paley's construction, p the
+ * smallest such order (odd part of r times 2^m, m >= 2, p - 1 prime) that divides r.
+ * A power of two has p = 1.  Returns 0 (and leaves *p, *k unchanged) when r admits
+ * neither. */
+int orc_tail_factor(int r, int* p, int* k) {
+    if (r <= 0) return 0;
+    if (is_pow2(r)) {
+        int t = 0;
+        while ((1 << t) < r) ++t;
+        *p = 1;
+        *k = t;
+        return 1;
+    }
+    int tz = 0;
+    while (((r >> tz) & 1) == 0) ++tz;
+    const int odd = r >> tz;
+    for (int m = 2; m <= tz; ++m) {
+        const long cand = (long)odd << m;
+        if (is_prime(cand - 1)) {
+            *p = (int)cand;
+            *k = tz - m;
+            return 1;
+        }
+    }
+    return 0;
+}
+
+/* Entry (i, j) of the tail block's Hadamard matrix H_p (x) H_(2^k) (r = p 2^k):
+ * H_p[i >> k][j >> k] * H_(2^k)[i & (2^k - 1)][j & (2^k - 1)]. */
+int orc_tail_entry(int r, int i, int j) {
+    int p, k;
+    if (!orc_tail_factor(r, &p, &k)) return 0;
+    if (p == 1) return orc_hadamard_entry(i, j);
+    const int mask = (1 << k) - 1;
+    return orc_paley_entry(p, i >> k, j >> k) * orc_hadamard_entry(i & mask, j & mask);
+}
+
 /* Block layout of R along K: q whole blocks of size B then one tail of size r.
- * Returns 0 when K does not split into blocks of B plus a power-of-two tail. */
+ * Returns 0 when K does not split into blocks of B plus a tail that is a power of two
+ * or a Paley order times a power of two (orc_tail_factor). */
 int orc_block_layout(int K, int B, int* q, int* r) {
     if (K <= 0 || !is_pow2(B)) return 0;
     *q = K / B;
     *r = K % B;
-    if (*r != 0 && !is_pow2(*r)) return 0;
+    int p, k;
+    if (*r != 0 && !orc_tail_factor(*r, &p, &k)) return 0;
     return 1;
 }
 
 /* y[k] = sum_j x[j] R[j][k] for one row of length K, in fp64.
- * R = blockdiag(H_B/sqrt(B), ..., H_r/sqrt(r)).  Returns 0 on a bad layout. */
+ * R = blockdiag(H_B/sqrt(B), ..., H_r/sqrt(r)), the tail's H_r from orc_tail_entry.
+ * Returns 0 on a bad layout. */
 int orc_rotate_row_f64(const double* x, double* y, int K, int B) {
     int q, r;
     if (!orc_block_layout(K, B, &q, &r)) return 0;
@@ -132,7 +208,8 @@ int orc_rotate_row_f64(const double* x, double* y, int K, int B) {
         double norm = sqrt((double)n);
         for (int k = 0; k < n; ++k) {
             double acc = 0.0;
-            for (int j = 0; j < n; ++j) acc += x[k0 + j] * (double)orc_hadamard_entry(j, k);
+            for (int j = 0; j < n; ++j)
+                acc += x[k0 + j] * (double)(b < q ? orc_hadamard_entry(j, k) : orc_tail_entry(n, j, k));
             y[k0 + k] = acc / norm;
         }
     }

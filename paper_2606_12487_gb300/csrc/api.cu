@@ -7,8 +7,11 @@
 #include <cstdio>
 #include <cstdlib>
 #include <cstring>
+#include <atomic>
 #include <map>
 #include <mutex>
+#include <set>
+#include <utility>
 #include <string>
 #include <vector>
 
@@ -230,6 +233,8 @@ dptq_status run_gemm(dptq_handle h, const GemmPlan& plan0, const uint8_t* act, c
   g.counters = sc->counters;
   g.gsync = sc->gsync;
   g.err = sc->err;
+  g.wait_cycles = wait_cycles_setting();
+  if (plan.fused) g.rq_shortfall = take_rows_shortfall();
   DPTQ_CUDA(launch_gemm(plan, s, true), "qgemm launch");
   return DPTQ_OK;
 }
@@ -259,6 +264,45 @@ bool l2_prefetch_allowed() {
     return !(v && v[0] == '0');
   }();
   return on;
+}
+
+long long wait_cycles_setting() {
+  static const long long v = [] {
+    const char* e = std::getenv("DPTQ_WAIT_CYCLES");
+    const long long c = e ? std::atoll(e) : 0LL;
+    return c > 0 ? c : 2000000000LL;
+  }();
+  return v;
+}
+
+int take_rows_shortfall() {
+  static std::atomic<int> left{[] {
+    const char* e = std::getenv("DPTQ_TEST_ROWS_SHORTFALL");
+    return e ? std::atoi(e) : 0;
+  }()};
+  return left.exchange(0);
+}
+
+cudaError_t ensure_max_dyn_smem_impl(const void* fn) {
+  // One entry per (kernel, device) whose ceiling is already raised.
+  static std::mutex mu;
+  static std::set<std::pair<const void*, int>> done;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  std::lock_guard<std::mutex> lk(mu);
+  if (done.count({fn, dev})) return cudaSuccess;
+  // The ceiling is the device's opt-in maximum per block less the kernel's static shared
+  // memory.
+  int optin = 0;
+  e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+  if (e != cudaSuccess) return e;
+  cudaFuncAttributes fa{};
+  e = cudaFuncGetAttributes(&fa, fn);
+  if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, optin - (int)fa.sharedSizeBytes);
+  if (e == cudaSuccess) done.insert({fn, dev});
+  return e;
 }
 
 bool rows_kernel_allowed() {

@@ -114,17 +114,17 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 }
 
 // Bounded wait for the phase of `parity` to complete.  Returns false if the CTA-wide
-// abort flag is raised or the wait times out (then the flag is raised and `code` is
-// recorded in the global error word).
+// abort flag is raised or the wait times out after `limit` cycles (then the flag is
+// raised and `code` is recorded in the global error word).
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
-                                          int* err, int code) {
+                                          int* err, int code, long long limit = kWaitTimeoutCycles) {
   if (mbar_try_wait(bar, parity)) return true;
   const long long t0 = clock64();
   while (true) {
     if (mbar_try_wait(bar, parity)) return true;
     __nanosleep(20);   // yield issue slots to the warps doing work
     if (*abort_flag) return false;
-    if (clock64() - t0 > kWaitTimeoutCycles) {
+    if (clock64() - t0 > limit) {
       *abort_flag = 1;
       atomicCAS(err, 0, code);
       return false;
@@ -137,14 +137,14 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
 // advance twice while the warp polls (true for every ring here: its next phase needs an
 // action of this warp first).
 __device__ __forceinline__ bool mbar_wait_warp(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
-                                               int* err, int code) {
+                                               int* err, int code, long long limit = kWaitTimeoutCycles) {
   if (__all_sync(0xffffffffu, mbar_try_wait(bar, parity))) return true;
   const long long t0 = clock64();
   while (true) {
     if (__all_sync(0xffffffffu, mbar_try_wait(bar, parity))) return true;
     __nanosleep(20);
     int stop = 0;
-    if ((threadIdx.x & 31) == 0) stop = *abort_flag ? 1 : (clock64() - t0 > kWaitTimeoutCycles ? 2 : 0);
+    if ((threadIdx.x & 31) == 0) stop = *abort_flag ? 1 : (clock64() - t0 > limit ? 2 : 0);
     stop = __shfl_sync(0xffffffffu, stop, 0);
     if (stop) {
       if (stop == 2 && (threadIdx.x & 31) == 0) {

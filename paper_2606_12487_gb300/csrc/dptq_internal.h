@@ -126,7 +126,9 @@ struct GemmArgs {
   RQArgs rq;
   int rq_np;           // parts per token row (1, 2 or 4): work item = row * rq_np + part
   int rq_items;        // M_pad * rq_np: the value the rows-ready counter reaches
+  int rq_shortfall;    // test hook: extra items the activation producer waits for (0)
   uint32_t* gsync;
+  long long wait_cycles;   // bound of every pipeline wait (SM cycles) before the kernel gives up
 };
 
 struct GemmPlan {
@@ -152,6 +154,13 @@ cudaError_t launch_gemm(const GemmPlan& plan, cudaStream_t s, bool pdl);
 bool pdl_allowed();
 // The fused decode kernel is used unless the environment sets DPTQ_FUSED=0.
 bool fused_allowed();
+// Bound of the GEMM kernels' pipeline waits in SM cycles: DPTQ_WAIT_CYCLES, else about
+// one second.  Tests of the time-out path shorten it.
+long long wait_cycles_setting();
+// Test hook: DPTQ_TEST_ROWS_SHORTFALL=n makes the first fused launch of the process wait
+// for n more published token rows than any CTA publishes, so that its bounded wait runs
+// out (returns n once, then 0).
+int take_rows_shortfall();
 // Decode GEMM launches prefetch their weight share into L2 unless DPTQ_L2PF=0.
 bool l2_prefetch_allowed();
 // The GEMM operand rows are rotated and quantized by the whole-row kernel (sums kept in
@@ -164,6 +173,19 @@ bool rows_kernel_allowed();
 // arrival counters (synchronous; no allocation).  *word = 0 when the scratch was never
 // set up on that device.
 cudaError_t static_scratch_check_reset(int dev, int* word);
+
+// Raise a kernel's ceiling for dynamic shared memory to the most the device allows it, once
+// per device.
+// Every launch of a kernel then fits its ceiling whatever size was launched last: a CUDA
+// graph that captured launches of one kernel with different shared-memory sizes (4- and
+// 8-bit plans) replays them, and a profiler that re-launches one of its nodes on its own
+// finds a ceiling that node fits.  (Setting the ceiling to each launch's own size made the
+// value left by the last captured launch govern such re-launches.)
+cudaError_t ensure_max_dyn_smem_impl(const void* fn);
+template <class Kernel>
+cudaError_t ensure_max_dyn_smem(Kernel* fn) {
+  return ensure_max_dyn_smem_impl(reinterpret_cast<const void*>(fn));
+}
 
 // Message returned by dptq_last_error_message() on the calling thread.
 void set_error_message(const std::string& m);

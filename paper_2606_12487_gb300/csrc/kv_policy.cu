@@ -486,7 +486,7 @@ cudaError_t launch_policy(const PolicyArgs& a, int num_sms, cudaStream_t s) {
   const long long items = (long long)a.L * a.T;
   if (a.d <= kPolMaxStagedD) {
     const int smem = kPolStages * 8 * a.d;
-    e = cudaFuncSetAttribute(policy_stats_staged_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    e = ensure_max_dyn_smem(policy_stats_staged_kernel);
     int per_sm = 0;
     if (e == cudaSuccess)
       e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, policy_stats_staged_kernel, kPolThreads, smem);

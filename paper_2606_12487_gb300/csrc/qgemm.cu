@@ -162,7 +162,9 @@ struct Smem {
   __device__ __forceinline__ uint8_t* slot(int s) const {
     return base + conv_slots * KPS * kConvBytes + s * slot_bytes;
   }
-  __device__ __forceinline__ uint8_t* act(int s, int h, int p) const { return slot(s) + (h * planes + p) * kActBytes; }
+  // Plane-major within a stage, so that a plane's KPS k-blocks are adjacent (one bulk copy
+  // when they are adjacent in global memory too).
+  __device__ __forceinline__ uint8_t* act(int s, int h, int p) const { return slot(s) + (p * KPS + h) * kActBytes; }
   __device__ __forceinline__ uint8_t* wpack(int s) const { return slot(s) + KPS * planes * kActBytes; }
   __device__ __forceinline__ uint8_t* end(int S) const { return slot(S); }
 };
@@ -307,11 +309,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
         while (true) {
           int st = 0;
           if (lane == 0) {
-            if (ld_acquire_gpu(a.gsync) >= (uint32_t)a.rq_items)
+            if (ld_acquire_gpu(a.gsync) >= (uint32_t)(a.rq_items + a.rq_shortfall))
               st = 1;
             else if (*abort_flag)
               st = 2;
-            else if (clock64() - t0 > kWaitTimeoutCycles) {
+            else if (clock64() - t0 > a.wait_cycles) {
               *abort_flag = 1;
               atomicCAS(a.err, 0, (int)kDevTimeoutGrid);
               st = 2;
@@ -347,7 +349,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
         const bool tg = kTraceStages > 10 && wprod && leader && g >= 8 && g < 11;   // clocked stages (trace builds)
         (void)tg;
         if (tg) DPTQ_TRACE_CLOCK(tr, 224 + 3 * (g - 8));
-        if (!mbar_wait_warp(&empty[s], rg.ph ^ 1u, abort_flag, a.err, kDevTimeoutEmpty)) {
+        if (!mbar_wait_warp(&empty[s], rg.ph ^ 1u, abort_flag, a.err, kDevTimeoutEmpty, a.wait_cycles)) {
           ok = false;
           break;
         }
@@ -361,10 +363,18 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
             if (g == S - 1) prefetch_share();
           } else {
             mbar_arrive_expect_tx(&afull[s], a_tx);
-#pragma unroll
-            for (int h = 0; h < KPS; ++h)
+            if (kb_stride == act_bytes) {
+              // One token tile: a plane's KPS k-blocks are contiguous in global memory and in
+              // the stage, so each plane is one copy (the bulk-copy engine's cost is largely
+              // per copy).
               for (int pl = 0; pl < a.planes; ++pl)
-                bulk_g2s(sm.act(s, h, pl), asrc + h * kb_stride + pl * plane_stride, act_bytes, &afull[s], pol_a);
+                bulk_g2s(sm.act(s, 0, pl), asrc + pl * plane_stride, KPS * act_bytes, &afull[s], pol_a);
+            } else {
+#pragma unroll
+              for (int h = 0; h < KPS; ++h)
+                for (int pl = 0; pl < a.planes; ++pl)
+                  bulk_g2s(sm.act(s, h, pl), asrc + h * kb_stride + pl * plane_stride, act_bytes, &afull[s], pol_a);
+            }
           }
           if (tg) DPTQ_TRACE_CLOCK(tr, 226 + 3 * (g - 8));
         }
@@ -401,7 +411,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
     while (iter.next(un)) {
       const int b = a.nbuf == 2 ? (u & 1) : 0;
       const uint32_t tpar = ((a.nbuf == 2 ? (u >> 1) : u) & 1) ^ 1;
-      if (!mbar_wait_warp(&tempty[b], tpar, abort_flag, a.err, kDevTimeoutTmemEmpty)) break;
+      if (!mbar_wait_warp(&tempty[b], tpar, abort_flag, a.err, kDevTimeoutTmemEmpty, a.wait_cycles)) break;
       tc_fence_after();
       uint32_t d = tmem_base + (uint32_t)(b * NT * a.segs);
       int seg_left = a.seg_iters - un.i0 % a.seg_iters;   // iterations left in this segment
@@ -413,12 +423,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
         const bool tgm = kTraceStages > 10 && leader && gm >= 8 && gm < 11;   // stages whose steps are clocked (trace builds)
         (void)tgm;
         if (tgm) DPTQ_TRACE_CLOCK(tr, 200 + 8 * (gm - 8));
-        if (!mbar_wait_warp(&afull[s], rg.ph, abort_flag, a.err, kDevTimeoutFull)) {
+        if (!mbar_wait_warp(&afull[s], rg.ph, abort_flag, a.err, kDevTimeoutFull, a.wait_cycles)) {
           ok = false;
           break;
         }
         if (tgm) DPTQ_TRACE_CLOCK(tr, 201 + 8 * (gm - 8));
-        if (!mbar_wait_warp(&cfull[c], rc.ph, abort_flag, a.err, kDevTimeoutConv)) {
+        if (!mbar_wait_warp(&cfull[c], rc.ph, abort_flag, a.err, kDevTimeoutConv, a.wait_cycles)) {
           ok = false;
           break;
         }
@@ -439,7 +449,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
 #pragma unroll
             for (int p = 0; p < 2; ++p) {
               if (p < planes) {
-                const uint64_t bd = bd_slot + (uint64_t)((h * planes + p) * act_step);
+                const uint64_t bd = bd_slot + (uint64_t)((p * KPS + h) * act_step);
 #pragma unroll
                 for (int ks = 0; ks < 4; ++ks) {   // 4 x (K = 32 FP8 elements = 32 bytes = 8 columns)
                   const uint32_t accumulate = (h | p | ks) ? 1u : (fresh ^ 1u);
@@ -530,12 +540,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
         // copy (stage gc - S, converted by the other group) is still in flight.  With
         // S >= CS, that copy has landed and been consumed once the MMA of stage gc - CS
         // is done.
-        if (gc >= CS && !mbar_wait(&empty[rl.s], rl.ph, abort_flag, a.err, kDevTimeoutConv)) {
+        if (gc >= CS && !mbar_wait(&empty[rl.s], rl.ph, abort_flag, a.err, kDevTimeoutConv, a.wait_cycles)) {
           ok = false;
           break;
         }
         if (tgc) DPTQ_TRACE_CLOCK(tr, 181 + 6 * (gc - 8));
-        if (!mbar_wait(&full[s], rg.ph, abort_flag, a.err, kDevTimeoutFull)) {
+        if (!mbar_wait(&full[s], rg.ph, abort_flag, a.err, kDevTimeoutFull, a.wait_cycles)) {
           ok = false;
           break;
         }
@@ -650,7 +660,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
     // ------------------------------------------------------------ epilogue
     pdl_wait();   // scales come from the previous kernel; `out` may still be read by it
     bool epi_ok = true;
-    if constexpr (FUSED) epi_ok = mbar_wait(aready, 0, abort_flag, a.err, kDevTimeoutGrid);
+    if constexpr (FUSED) epi_ok = mbar_wait(aready, 0, abort_flag, a.err, kDevTimeoutGrid, a.wait_cycles);
     const float* __restrict__ sa_g = a.sa;
     const float* __restrict__ sw_g = a.sw;
     __half* __restrict__ out_g = a.out;
@@ -665,7 +675,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
     auto epi_sync = [&]() -> bool {
       __syncwarp();
       if (lane == 0) mbar_arrive(esync);
-      const bool ok = mbar_wait(esync, (uint32_t)(esync_phase & 1), abort_flag, a.err, kDevTimeoutTmemFull);
+      const bool ok = mbar_wait(esync, (uint32_t)(esync_phase & 1), abort_flag, a.err, kDevTimeoutTmemFull, a.wait_cycles);
       ++esync_phase;
       return ok;
     };
@@ -691,7 +701,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
         if (!epi_sync()) break;
         sa_mt = mt;
       }
-      if (!mbar_wait(&tfull[b], tpar, abort_flag, a.err, kDevTimeoutTmemFull)) break;
+      if (!mbar_wait(&tfull[b], tpar, abort_flag, a.err, kDevTimeoutTmemFull, a.wait_cycles)) break;
       if (etid == 0 && u < 4) DPTQ_TRACE_POINT(tr, 104 + u);
       tc_fence_after();
       const int nseg = (un.i1 - 1) / a.seg_iters - un.i0 / a.seg_iters + 1;
@@ -1082,13 +1092,14 @@ bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan, i
   }
   a.rq_np = np;
   a.rq_items = fused ? M_pad * np : 0;
+  a.rq_shortfall = 0;
+  a.wait_cycles = kWaitTimeoutCycles;
   return true;
 }
 
 template <int NT, int KPS, int RQV = 0>
 static cudaError_t launch_nt(const GemmPlan& plan, cudaStream_t s, bool pdl) {
-  cudaError_t e = cudaFuncSetAttribute(qgemm_kernel<NT, KPS, RQV>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       plan.smem_bytes);
+  cudaError_t e = ensure_max_dyn_smem(qgemm_kernel<NT, KPS, RQV>);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)plan.grid);

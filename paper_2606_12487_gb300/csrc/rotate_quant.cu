@@ -220,7 +220,7 @@ cudaError_t launch_rotate_quant(RQMode mode, const RQArgs& a, cudaStream_t s, bo
   cudaError_t e = cudaSuccess;
   switch (mode) {
     case kRQPublic:
-      e = cudaFuncSetAttribute(rotate_quant_kernel<kRQPublic>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      e = ensure_max_dyn_smem(rotate_quant_kernel<kRQPublic>);
       if (e == cudaSuccess) e = cudaLaunchKernelEx(&cfg, rotate_quant_kernel<kRQPublic>, a);
       break;
     case kRQAct: {
@@ -228,37 +228,36 @@ cudaError_t launch_rotate_quant(RQMode mode, const RQArgs& a, cudaStream_t s, bo
       if (nch >= 1 && rows_kernel_allowed()) {
         cfg.blockDim = dim3(kRQThreads * nch);
         cfg.dynamicSmemBytes = (size_t)nch * kChunkPadded * 8;
-        const int sm = (int)cfg.dynamicSmemBytes;
         switch (nch) {
           case 1:
-            e = cudaFuncSetAttribute(rotate_quant_rows_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+            e = ensure_max_dyn_smem(rotate_quant_rows_kernel<1>);
             if (e == cudaSuccess) e = cudaLaunchKernelEx(&cfg, rotate_quant_rows_kernel<1>, a);
             break;
           case 2:
-            e = cudaFuncSetAttribute(rotate_quant_rows_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+            e = ensure_max_dyn_smem(rotate_quant_rows_kernel<2>);
             if (e == cudaSuccess) e = cudaLaunchKernelEx(&cfg, rotate_quant_rows_kernel<2>, a);
             break;
           case 3:
-            e = cudaFuncSetAttribute(rotate_quant_rows_kernel<3>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+            e = ensure_max_dyn_smem(rotate_quant_rows_kernel<3>);
             if (e == cudaSuccess) e = cudaLaunchKernelEx(&cfg, rotate_quant_rows_kernel<3>, a);
             break;
           default:
-            e = cudaFuncSetAttribute(rotate_quant_rows_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+            e = ensure_max_dyn_smem(rotate_quant_rows_kernel<4>);
             if (e == cudaSuccess) e = cudaLaunchKernelEx(&cfg, rotate_quant_rows_kernel<4>, a);
             break;
         }
         break;
       }
-      e = cudaFuncSetAttribute(rotate_quant_kernel<kRQAct>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      e = ensure_max_dyn_smem(rotate_quant_kernel<kRQAct>);
       if (e == cudaSuccess) e = cudaLaunchKernelEx(&cfg, rotate_quant_kernel<kRQAct>, a);
       break;
     }
     case kRQY:
-      e = cudaFuncSetAttribute(rotate_quant_kernel<kRQY>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      e = ensure_max_dyn_smem(rotate_quant_kernel<kRQY>);
       if (e == cudaSuccess) e = cudaLaunchKernelEx(&cfg, rotate_quant_kernel<kRQY>, a);
       break;
     case kRQWeights:
-      e = cudaFuncSetAttribute(rotate_quant_kernel<kRQWeights>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      e = ensure_max_dyn_smem(rotate_quant_kernel<kRQWeights>);
       if (e == cudaSuccess) e = cudaLaunchKernelEx(&cfg, rotate_quant_kernel<kRQWeights>, a);
       break;
   }

@@ -112,3 +112,45 @@ def test_injected_allocation_failure_reports_oom(fail_at, expect):
     and token scales."""
     out = _child(CHILD, fail_at).strip().splitlines()[-1]
     assert out == expect, out
+
+
+TIMEOUT_CHILD = """
+import torch
+from paper_2606_12487_gb300 import dptq, inputs
+lib = dptq.load()
+M, K, N = 32, 4096, 4096
+W = torch.from_numpy(inputs.weights(N, K, layer=1)).cuda()
+x = torch.from_numpy(inputs.activations(inputs.llama2_7b_decode(), M, K)).cuda()
+layer = dptq.dptq_pack_weights(W, 4096)
+ref = torch.empty((M, N), dtype=torch.float16, device="cuda")
+dptq.dptq_qlinear_quantize(layer, x, 4)
+dptq.dptq_qlinear_gemm(layer, M, 4, ref)     # two launches: untouched by the hook
+torch.cuda.synchronize()
+assert lib.dptq_last_device_error(None) == 0
+out = torch.zeros_like(ref)
+dptq.dptq_qlinear(layer, x, 4, out)          # first fused launch: waits for a row that never comes
+torch.cuda.synchronize()
+st1 = lib.dptq_last_device_error(None)
+msg = lib.dptq_last_error_message().decode()
+dptq.dptq_qlinear(layer, x, 4, out)          # the next launch runs normally
+torch.cuda.synchronize()
+st2 = lib.dptq_last_device_error(None)
+same = torch.equal(out.view(torch.int16), ref.view(torch.int16))
+print(st1, st2, "same" if same else "differs", "|", msg)
+"""
+
+
+def test_bounded_wait_times_out_and_recovers():
+    """A fused launch is made to wait for one more published token row than its CTAs
+    publish (host-side test hook), with the wait bound shortened to 200k cycles (~0.1 ms).
+    Every CTA's bounded wait runs out: the kernel records the time-out, drains its own
+    copies, frees its tensor memory and returns, and dptq_last_device_error reports
+    DPTQ_ERR_TIMEOUT and clears the scratch.  The next launch is then bit-identical to
+    the two-launch path.  No GPU fault is involved: the wait ends by its bound."""
+    env = dict(os.environ, DPTQ_WAIT_CYCLES="200000", DPTQ_TEST_ROWS_SHORTFALL="1")
+    r = subprocess.run([sys.executable, "-c", textwrap.dedent(TIMEOUT_CHILD)], cwd=ROOT, env=env,
+                       capture_output=True, text=True, timeout=600)
+    assert r.returncode == 0, r.stdout + r.stderr
+    line = r.stdout.strip().splitlines()[-1]
+    assert line.startswith("5 0 same"), line
+    assert "timed out" in line

@@ -462,3 +462,80 @@ def test_policy_mask_closed_form(orc):
     assert bits.tolist() == [8, 4, 4, 4, 8, 4]
     assert orc.policy_mask(jr, snr, tau_jr=-1.0, tau_snr=1e9).tolist() == [8] * 6
     assert orc.policy_mask(jr, snr, tau_jr=1.0, tau_snr=1e9).tolist() == [4] * 6
+
+
+# ---------------------------------------------------------------- non-power-of-two tail blocks
+def test_paley_h12_golden(orc):
+    """Rows 0 and 1 of Paley's H_12 and the quadratic character mod 11, worked by hand."""
+    chi, row0, row1 = ([int(v) for v in ln.split()] for ln in _rows("paley_q11.txt"))
+    assert [orc.paley_entry(12, 0, j) for j in range(12)] == row0
+    assert [orc.paley_entry(12, 1, j) for j in range(12)] == row1
+    assert [orc.paley_entry(12, 1, 1 + a) for a in range(1, 11)] == chi
+
+
+@pytest.mark.parametrize("p", [12, 20, 24, 44, 48, 60, 68, 72, 80, 84])
+def test_paley_matrices_are_hadamard(orc, p):
+    """H_p H_p^T = p I exactly, H_p = I + S with S skew-symmetric, first row all ones
+    (Paley's first construction for the prime p - 1 = 3 mod 4)."""
+    H = np.array([[orc.paley_entry(p, i, j) for j in range(p)] for i in range(p)], dtype=np.int64)
+    assert np.array_equal(H @ H.T, p * np.eye(p, dtype=np.int64))
+    S = H - np.eye(p, dtype=np.int64)
+    assert np.array_equal(S.T, -S)
+    assert np.all(H[0] == 1) and np.all(np.abs(H) == 1)
+
+
+def test_paley_entry_rejects_other_orders(orc):
+    for p in (10, 16, 28, 36, 52):   # not a multiple of 4, or p - 1 composite (15, 27, 35, 51)
+        assert orc.paley_entry(p, 1, 2) == 0
+
+
+@pytest.mark.parametrize("r,expect", [(2816, (44, 6)), (1536, (12, 7)), (512, (1, 9)), (96, (12, 3)),
+                                      (160, (20, 3)), (6, None), (3, None), (44, (44, 0))])
+def test_tail_factor(orc, r, expect):
+    assert orc.tail_factor(r) == expect
+
+
+@pytest.mark.parametrize("r", [12 * 16, 44 * 4, 20 * 8, 2816])
+def test_tail_block_is_kronecker_and_orthogonal(orc, r):
+    """The tail block's matrix is H_p (x) H_(2^k) (numpy's kron of the two factors) and is a
+    Hadamard matrix of order r."""
+    p, k = orc.tail_factor(r)
+    Hp = np.array([[orc.paley_entry(p, i, j) for j in range(p)] for i in range(p)], dtype=np.int64)
+    ref = np.kron(Hp, sylvester(1 << k))
+    idx = range(r) if r <= 256 else np.random.default_rng(r).choice(r, 96, replace=False)
+    for i in idx:
+        assert [orc.tail_entry(r, int(i), j) for j in range(r)] == ref[int(i)].tolist()
+    assert np.array_equal(ref @ ref.T, r * np.eye(r, dtype=np.int64))
+
+
+@pytest.mark.parametrize("K,B", [(256 + 192, 256), (1024 + 176, 1024), (4096 + 2816, 4096)])
+def test_rotation_with_paley_tail_is_orthogonal(orc, K, B):
+    """R^T R = I (Section 2 Eq. 4) with a non-power-of-two tail: the rotated basis rows are
+    orthonormal, norms are kept, and the tail block equals x_tail H_r / sqrt(r)."""
+    q, r = orc.block_layout(K, B)
+    assert r == K - q * B and orc.tail_factor(r)[0] > 1
+    rng = np.random.default_rng(K)
+    for _ in range(3):
+        x = rng.standard_normal(K)
+        y = orc.rotate_row_f64(x, B)
+        assert abs(np.linalg.norm(y) - np.linalg.norm(x)) < 1e-10 * np.linalg.norm(x)
+    p, k = orc.tail_factor(r)
+    Hp = np.array([[orc.paley_entry(p, i, j) for j in range(p)] for i in range(p)], dtype=np.float64)
+    Hr = np.kron(Hp, sylvester(1 << k).astype(np.float64))
+    x = rng.standard_normal(K)
+    y = orc.rotate_row_f64(x, B)
+    assert np.allclose(y[q * B:], x[q * B:] @ Hr / math.sqrt(r), rtol=0, atol=1e-12)
+    if K <= 1200:
+        R = np.array([orc.rotate_row_f64(e, B) for e in np.eye(K)])
+        assert np.allclose(R @ R.T, np.eye(K), atol=1e-12)
+
+
+def test_fold_equivalence_with_paley_tail(orc):
+    """Eq. 5 with a non-power-of-two tail: (X R)(W R)^T = X W^T."""
+    K, B = 256 + 96, 256
+    rng = np.random.default_rng(5)
+    X = rng.standard_normal((3, K))
+    W = rng.standard_normal((4, K))
+    XR = np.array([orc.rotate_row_f64(x, B) for x in X])
+    WR = np.array([orc.rotate_row_f64(w, B) for w in W])
+    assert np.allclose(XR @ WR.T, X @ W.T, atol=1e-10)
