@@ -17,8 +17,12 @@
  *
  * Numerics (readings where the paper is silent):
  *   R = blockdiag(H_B, ..., H_B, H_r) / sqrt(block) along K, H the Sylvester
- *   Hadamard matrix in natural order, B = had_block a power of two, r = K mod B a
- *   power of two (or 0).  Scales s = max|row| / (2^(b-1) - 1) in fp32 (IEEE
+ *   Hadamard matrix in natural order, B = had_block a power of two, r = K mod B.
+ *   A tail r that is not a power of two takes H_r = H_p (x) H_(2^k) with r = p 2^k
+ *   and H_p the Paley type-I matrix of order p (p - 1 prime, p = 3 mod 4; the
+ *   smallest such p, so that 2^k is largest), H_p = I + S, S[0][j>0] = 1, S[i>0][0] = -1,
+ *   S[i][j] = chi(j - i) for i, j >= 1 with chi the quadratic character mod p - 1
+ *   (Paley's first construction); the tail is scaled by 1/sqrt(r).  Scales s = max|row| / (2^(b-1) - 1) in fp32 (IEEE
  *   division); codes round half to even, clamped to [-2^(b-1), 2^(b-1) - 1];
  *   an all-zero row has s = 0 and all codes 0.  Output
  *   out[m][n] = fp16_rne( fp32( fp32(acc[m][n]) * s_a[m] ) * s_w[n] ).
@@ -34,8 +38,11 @@
  *     host.  Calls that share one handle, or the library scratch of one device,
  *     must not run concurrently on different streams.
  *   - Shape rules: 1 <= K <= 49152, K % 32 == 0, N % 16 == 0, had_block a power of
- *     two <= 4096, K splits into blocks of had_block plus a power-of-two tail, bits in
- *     {4, 8}.  Violations return
+ *     two <= 4096, K splits into blocks of had_block plus a tail r that is a power of
+ *     two or p 2^k with a Paley order p <= 256 (r = 2816 = 44 x 64 at K = 11008 and
+ *     had_block 4096; r = 96 = 12 x 8, but not r = 736 = 23 x 32), bits in {4, 8}.
+ *     Layers with a non-power-of-two tail run dptq_qlinear as two launches
+ *     (rotate-quantize, then GEMM); dptq_qlinear_static rejects them.  Violations return
  *     DPTQ_ERR_INVALID_ARG (bits, null pointers, negative sizes) or
  *     DPTQ_ERR_UNSUPPORTED (shape).  M == 0 is a no-op.
  *   - No exception crosses this boundary.  CUDA errors map to DPTQ_ERR_CUDA (failed
@@ -188,7 +195,8 @@ dptq_status dptq_qlinear_gemm(dptq_handle h, int M, int bits, void* out_fp16, vo
  * device array of about 5 MiB inside the library, which every GPU that loads the
  * library holds until the process exits.  The call never runs cudaMalloc, cudaFree or
  * an allocating library routine.
- * Limits: M <= 32 tokens and K <= 16384; larger shapes return DPTQ_ERR_UNSUPPORTED.
+ * Limits: M <= 32 tokens, K <= 16384 and a power-of-two tail block (K mod had_block);
+ * other shapes return DPTQ_ERR_UNSUPPORTED.
  * The first call on a device looks the array up (cudaGetSymbolAddress) and zeroes it,
  * synchronously; make that first call before any stream capture.  That first call is
  * also when the CUDA driver brings the array's device memory in (modules load lazily),

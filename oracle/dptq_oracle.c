@@ -195,10 +195,23 @@ int orc_block_layout(int K, int B, int* q, int* r) {
     return 1;
 }
 
+/* The tail block's matrix H_r as a table, tab[j * r + k] = orc_tail_entry(r, j, k), when
+ * the tail r = K mod B is not a power of two (its entries then cost a primality test and
+ * a Legendre symbol each); NULL otherwise, and the entries are taken one by one. */
+static signed char* tail_table(int K, int B) {
+    int q, r, p, k;
+    if (!orc_block_layout(K, B, &q, &r) || r == 0 || is_pow2(r) || !orc_tail_factor(r, &p, &k)) return NULL;
+    signed char* tab = (signed char*)malloc((size_t)r * (size_t)r);
+    if (!tab) return NULL;
+    for (int j = 0; j < r; ++j)
+        for (int c = 0; c < r; ++c) tab[(size_t)j * r + c] = (signed char)orc_tail_entry(r, j, c);
+    return tab;
+}
+
 /* y[k] = sum_j x[j] R[j][k] for one row of length K, in fp64.
- * R = blockdiag(H_B/sqrt(B), ..., H_r/sqrt(r)), the tail's H_r from orc_tail_entry.
- * Returns 0 on a bad layout. */
-int orc_rotate_row_f64(const double* x, double* y, int K, int B) {
+ * R = blockdiag(H_B/sqrt(B), ..., H_r/sqrt(r)), the tail's H_r from orc_tail_entry
+ * (read from tab when given).  Returns 0 on a bad layout. */
+static int rotate_row(const double* x, double* y, int K, int B, const signed char* tab) {
     int q, r;
     if (!orc_block_layout(K, B, &q, &r)) return 0;
     int nblk = q + (r ? 1 : 0);
@@ -208,12 +221,22 @@ int orc_rotate_row_f64(const double* x, double* y, int K, int B) {
         double norm = sqrt((double)n);
         for (int k = 0; k < n; ++k) {
             double acc = 0.0;
-            for (int j = 0; j < n; ++j)
-                acc += x[k0 + j] * (double)(b < q ? orc_hadamard_entry(j, k) : orc_tail_entry(n, j, k));
+            for (int j = 0; j < n; ++j) {
+                const int h = b < q ? orc_hadamard_entry(j, k)
+                                    : (tab ? tab[(size_t)j * n + k] : orc_tail_entry(n, j, k));
+                acc += x[k0 + j] * (double)h;
+            }
             y[k0 + k] = acc / norm;
         }
     }
     return 1;
+}
+
+int orc_rotate_row_f64(const double* x, double* y, int K, int B) {
+    signed char* tab = tail_table(K, B);
+    const int ok = rotate_row(x, y, K, B, tab);
+    free(tab);
+    return ok;
 }
 
 /* Rotate an fp16 matrix x[M][K] (row-major, raw binary16 bits) into fp32 y[M][K]:
@@ -228,14 +251,16 @@ int orc_rotate_f16_signed(const uint16_t* x, float* y, int M, int K, int B, cons
     double* xr = (double*)malloc(sizeof(double) * (size_t)K);
     double* yr = (double*)malloc(sizeof(double) * (size_t)K);
     if (!xr || !yr) { free(xr); free(yr); return 0; }
+    signed char* tab = tail_table(K, B);
     for (int m = 0; m < M; ++m) {
         for (int k = 0; k < K; ++k) {
             xr[k] = orc_half_to_double(x[(size_t)m * K + k]);
             if (signs && signs[k] < 0) xr[k] = -xr[k];
         }
-        orc_rotate_row_f64(xr, yr, K, B);
+        rotate_row(xr, yr, K, B, tab);
         for (int k = 0; k < K; ++k) y[(size_t)m * K + k] = (float)yr[k];
     }
+    free(tab);
     free(xr);
     free(yr);
     return 1;

@@ -42,12 +42,46 @@ dptq_status cuda_fail(cudaError_t e, const char* where) {
 
 bool is_pow2(int v) { return v > 0 && (v & (v - 1)) == 0; }
 
-// Block layout of R along K: nfull blocks of B then a power-of-two tail (or none).
+bool is_prime_int(int v) {
+  if (v < 2) return false;
+  for (int d = 2; d * d <= v; ++d)
+    if (v % d == 0) return false;
+  return true;
+}
+
+// A tail block of r elements is r = p 2^k: p = 1 for a power of two; otherwise p is the
+// smallest Paley order (odd part of r times 2^m, m >= 2, with p - 1 prime) that divides r,
+// and the tail's Hadamard matrix is H_p (x) H_(2^k) with H_p from Paley's first
+// construction.  False when r is neither.
+bool tail_factor(int r, int& p, int& k) {
+  if (r <= 0) return false;
+  if (is_pow2(r)) {
+    p = 1;
+    k = 0;
+    while ((1 << k) < r) ++k;
+    return true;
+  }
+  int tz = 0;
+  while (((r >> tz) & 1) == 0) ++tz;
+  const int odd = r >> tz;
+  for (int m = 2; m <= tz; ++m) {
+    if (is_prime_int((odd << m) - 1)) {
+      p = odd << m;
+      k = tz - m;
+      return true;
+    }
+  }
+  return false;
+}
+
+// Block layout of R along K: nfull blocks of B then a tail (or none) that is a power of
+// two or a Paley order times a power of two.
 bool hadamard_layout(int K, int B, int& nfull, int& tail, int& log2B) {
   if (!is_pow2(B) || K <= 0) return false;
   nfull = K / B;
   tail = K % B;
-  if (tail != 0 && !is_pow2(tail)) return false;
+  int p, k;
+  if (tail != 0 && !tail_factor(tail, p, k)) return false;
   log2B = 0;
   while ((1 << log2B) < B) ++log2B;
   return true;
@@ -60,11 +94,25 @@ int rq_chunk(int K, int B) {
   return c < K ? c : K;
 }
 
+// Whether K's tail block is a power of two (or absent); the fused decode launch and the
+// whole-row kernel handle only those.
+bool pow2_tail(int K, int B) { return K % B == 0 || is_pow2(K % B); }
+
 dptq_status check_shape(int K, int B, int& nfull, int& tail, int& log2B) {
   if (K % 32 != 0) return fail(DPTQ_ERR_UNSUPPORTED, "K must be a multiple of 32");
   if (B > 4096) return fail(DPTQ_ERR_UNSUPPORTED, "had_block above 4096 is not supported");
   if (!hadamard_layout(K, B, nfull, tail, log2B))
-    return fail(DPTQ_ERR_UNSUPPORTED, "K must split into blocks of had_block (a power of two) plus a power-of-two tail");
+    return fail(DPTQ_ERR_UNSUPPORTED,
+                "K must split into blocks of had_block (a power of two) plus a tail that is a power of two or a "
+                "Paley order times a power of two");
+  int p = 1, k = 0;
+  if (tail != 0 && !is_pow2(tail)) {
+    tail_factor(tail, p, k);
+    if (p > 256) return fail(DPTQ_ERR_UNSUPPORTED, "the tail block's Paley order is above 256");
+    // The tail must lie in the last 4096-element rotation pass.
+    if (nfull * B < ((K - 1) / 4096) * 4096)
+      return fail(DPTQ_ERR_UNSUPPORTED, "a non-power-of-two tail must lie in the last 4096 elements of K");
+  }
   if (rotate_quant_smem(K, rq_chunk(K, B)) > kSmemPerBlock)
     return fail(DPTQ_ERR_UNSUPPORTED, "K and had_block exceed the shared memory of one CTA");
   return DPTQ_OK;
@@ -83,7 +131,19 @@ RQArgs make_rq(const void* x, int rows_in, int rows_out, int K, int KB, int B, i
   a.nfull = nfull;
   a.tail = tail;
   a.log2T = 0;
-  while (tail && (1 << a.log2T) < tail) ++a.log2T;
+  a.tail_p = 1;
+  a.tail_j = 0;
+  int p = 1, k = 0;
+  if (tail && tail_factor(tail, p, k)) {
+    a.log2T = k;
+    a.tail_p = p;
+    if (p > 1) {   // y = S 2^-24 / sqrt(p 2^k) = S 2^-(24 + k/2) / sqrt(p 2^(k mod 2))
+      const double t = 1.0 / std::sqrt((double)p * (double)(1 << (k & 1)));
+      a.tail_j = k >> 1;
+      a.t_hi = (float)t;
+      a.t_lo = (float)(t - (double)a.t_hi);
+    }
+  }
   a.chunk = rq_chunk(K, B);
   const double r2 = 1.0 / std::sqrt(2.0);
   a.c_hi = (float)r2;
@@ -509,7 +569,7 @@ dptq_status dptq_qlinear(dptq_handle h, const void* x_fp16, int M, int bits, voi
   if (!x_fp16 || !out_fp16) return fail(DPTQ_ERR_INVALID_ARG, "null pointer");
   // Small M: one launch that rotates and quantizes the rows and runs the GEMM.
   GemmPlan fp;
-  if (fused_allowed() && h->K_pad <= kFusedMaxKPad &&
+  if (fused_allowed() && h->K_pad <= kFusedMaxKPad && pow2_tail(h->K, h->had_block) &&
       plan_gemm(M, h->N, h->K_pad, bits, sc->num_sms, fp, kRQPartSmemBytes) && fp.M_pad == plan.M_pad) {
     int nfull, tail, log2B;
     if ((st = check_shape(h->K, h->had_block, nfull, tail, log2B)) != DPTQ_OK) return st;

@@ -51,6 +51,13 @@ struct RQArgs {
   int log2T;         // log2(tail) (0 when there is no tail)
   int chunk;         // elements rotated per shared-memory pass (a multiple of B)
   float c_hi, c_lo;  // 1/sqrt(2) as an fp32 pair (c_hi + c_lo to ~2^-48)
+  // Non-power-of-two tail block r = tail_p 2^log2T (tail_p > 1): H_p (x) H_(2^log2T), H_p
+  // from Paley's first construction with the prime tail_p - 1; y = S 2^-(24 + tail_j)
+  // (t_hi + t_lo), t the fp32 pair of 1/sqrt(tail_p 2^(log2T & 1)).  tail_p = 1: a
+  // power-of-two tail (or none).
+  int tail_p;
+  int tail_j;
+  float t_hi, t_lo;
   int bits;          // 4 or 8
   float* scales;     // [rows_out] (rows >= rows_in get 0); may be null in kRQY
   void* out;         // mode-dependent destination

@@ -195,14 +195,15 @@ __global__ void __launch_bounds__(kRQThreads * NCH, NCH == 1 ? 3 : 1) rotate_qua
 // Whole-row kernel for the GEMM operand when the row fits in registers (K <= 16384, one
 // group of 256 threads per 4096-element chunk); -1 when it does not apply.
 int rows_kernel_chunks(const RQArgs& a) {
-  if (a.B > kChunk || a.K > 4 * kChunk) return -1;
+  if (a.B > kChunk || a.K > 4 * kChunk || a.tail_p > 1) return -1;
   const int nch = (a.K + kChunk - 1) / kChunk;
   return nch;
 }
 
 size_t rotate_quant_smem(int K, int chunk) {
   (void)chunk;
-  return (size_t)K * sizeof(float) + (size_t)kChunkPadded * sizeof(long long);
+  // the fp32 row, the int64 transpose chunk, and a Paley tail's character table (<= 256 B)
+  return (size_t)K * sizeof(float) + (size_t)kChunkPadded * sizeof(long long) + 256;
 }
 
 cudaError_t launch_rotate_quant(RQMode mode, const RQArgs& a, cudaStream_t s, bool pdl) {

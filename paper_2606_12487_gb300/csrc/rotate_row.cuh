@@ -135,15 +135,13 @@ __device__ __forceinline__ void apply_signs(const int8_t* sg, long long (&f)[16]
     if ((w[e >> 2] >> (8 * (e & 3) + 7)) & 1u) f[e] = -f[e];
 }
 
-// Correctly rounded fp32 of S * 2^-24 / sqrt(2^log2n) for an exact Hadamard sum S.
-// Even log2n: one rounding of S, then an exact power-of-two scale.  Odd log2n: S and
-// 1/sqrt(2) as fp32 pairs, the product formed with fma to ~2^-47 relative, and one
-// final rounding.
-__device__ __forceinline__ float fixed_to_rotated(long long S, int log2n, float c_hi, float c_lo) {
-  const int j = log2n >> 1;
+// fp32 of S * 2^-(24 + j) * c for an exact sum S and an fp32 pair c = c_hi + c_lo (an
+// irrational constant to ~2^-48): S and c as fp32 pairs, their product formed with fma to
+// ~2^-47 relative, and one final rounding (correctly rounded except within ~2^-47 of a
+// rounding boundary).
+__device__ __forceinline__ float fixed_times_const(long long S, int j, float c_hi, float c_lo) {
   const float scale = __int_as_float((127 - 24 - j) << 23);   // 2^-(24 + j), exact
   const float hi = ll_to_float_rn(S);
-  if ((log2n & 1) == 0) return __fmul_rn(hi, scale);
   // S - hi exactly: hi = +-(1.f) * 2^e with e <= 52 is the integer mag << (e - 23); the
   // remainder is below 2^29 in magnitude.
   const uint32_t hb = __float_as_uint(hi);
@@ -159,6 +157,15 @@ __device__ __forceinline__ float fixed_to_rotated(long long S, int log2n, float 
   const float err = __fmaf_rn(hi, c_hi, -p);
   const float t = __fmaf_rn(hi, c_lo, __fmaf_rn(lo, c_hi, err));
   return __fmul_rn(__fadd_rn(p, t), scale);
+}
+
+// Correctly rounded fp32 of S * 2^-24 / sqrt(2^log2n) for an exact Hadamard sum S.
+// Even log2n: one rounding of S, then an exact power-of-two scale.  Odd log2n: the
+// product with 1/sqrt(2) (c_hi + c_lo) of fixed_times_const.
+__device__ __forceinline__ float fixed_to_rotated(long long S, int log2n, float c_hi, float c_lo) {
+  const int j = log2n >> 1;
+  if ((log2n & 1) == 0) return __fmul_rn(ll_to_float_rn(S), __int_as_float((127 - 24 - j) << 23));
+  return fixed_times_const(S, j, c_hi, c_lo);
 }
 
 // The row is rotated in chunks of 4096 elements (whole Hadamard blocks; the last chunk
@@ -196,12 +203,37 @@ __device__ __forceinline__ void rotate_quant_row(const RQArgs& a, int row, unsig
   const int tail_start = a.nfull << a.log2B;   // first element of the tail block
   float lmax = 0.f;   // this thread's largest |y|
 
+  // Non-power-of-two tail (tail_p > 1): the quadratic character mod q = tail_p - 1, one
+  // byte per residue, after the transpose buffer; the tail's sums wait in sx until every
+  // segment's H_(2^log2T) butterflies are done, then H_p mixes the segments.
+  const bool ptail = a.tail_p > 1;
+  signed char* chi = reinterpret_cast<signed char*>(smem + (size_t)K * sizeof(float) + (size_t)kChunkPadded * 8);
+  if (live && ptail) {
+    const int q = a.tail_p - 1;
+    for (int d = tid; d < q; d += kRQThreads) {
+      int r = 1, b = d, e = (q - 1) / 2;   // d^((q-1)/2) mod q (Euler's criterion)
+      while (e) {
+        if (e & 1) r = (r * b) % q;
+        b = (b * b) % q;
+        e >>= 1;
+      }
+      chi[d] = d == 0 ? 0 : (r == 1 ? 1 : -1);
+    }
+  }
+
   if (live) {
     const uint4* src = reinterpret_cast<const uint4*>(a.x + (size_t)row * K);
     for (int c0 = 0; c0 < K; c0 += kChunk) {
       const int len = min(kChunk, K - c0);
       // log2 of the block size that element i of this chunk belongs to
       auto lg = [&](int i) { return (c0 + i < tail_start) ? a.log2B : a.log2T; };
+      // fp32 of the sum of element c0 + i into sy (a Paley tail's sums are mixed later)
+      auto put = [&](long long S, int i) {
+        if (ptail && c0 + i >= tail_start) return;
+        const float yv = fixed_to_rotated(S, lg(i), a.c_hi, a.c_lo);
+        lmax = fmaxf(lmax, fabsf(yv));
+        sy[c0 + i] = yv;
+      };
       long long f[16];
       // ---- round A: load 16 consecutive fp16 values
       {
@@ -312,34 +344,59 @@ __device__ __forceinline__ void rotate_quant_row(const RQArgs& a, int row, unsig
 #pragma unroll
             for (int e = 0; e < 16; ++e) {
               const int i = 256 * e + tid;
-              if (i < len) {
-                const float yv = fixed_to_rotated(f[e], lg(i), a.c_hi, a.c_lo);
-                lmax = fmaxf(lmax, fabsf(yv));
-                sy[c0 + i] = yv;
-              }
+              if (i < len) put(f[e], i);
             }
           }
         } else {
 #pragma unroll
           for (int e = 0; e < 16; ++e) {
             const int i = iB + 16 * e;
-            if (i < len) {
-              const float yv = fixed_to_rotated(f[e], lg(i), a.c_hi, a.c_lo);
-              lmax = fmaxf(lmax, fabsf(yv));
-              sy[c0 + i] = yv;
-            }
+            if (i < len) put(f[e], i);
           }
         }
       } else {
 #pragma unroll
         for (int e = 0; e < 16; ++e) {
           const int i = iA + e;
-          if (i < len) {
-            const float yv = fixed_to_rotated(f[e], lg(i), a.c_hi, a.c_lo);
-            lmax = fmaxf(lmax, fabsf(yv));
-            sy[c0 + i] = yv;
-          }
+          if (i < len) put(f[e], i);
         }
+      }
+      if (ptail && c0 + len > tail_start) {
+        // The tail lies in this (last) chunk: park its sums, in tail order, in sx once
+        // every thread's transpose reads are done.
+        sync();
+        long long* tz = sx;
+#pragma unroll
+        for (int e = 0; e < 16; ++e) {
+          const int i = maxlg > 8 ? 256 * e + tid : maxlg > 4 ? 256 * (tid >> 4) + 16 * e + (tid & 15) : iA + e;
+          if (i < len && c0 + i >= tail_start) tz[c0 + i - tail_start] = f[e];
+        }
+      }
+    }
+    if (ptail) {
+      // y[a' 2^k + b'] = sum_a H_p[a][a'] z[a 2^k + b'] (exact), H_p[a][a'] = 1 on the
+      // diagonal and in row 0, -1 in column 0, chi(a' - a) elsewhere (Paley I); then
+      // y 2^-(24 + tail_j) (t_hi + t_lo) = S 2^-24 / sqrt(r).
+      sync();
+      const long long* tz = sx;
+      const int r = K - tail_start, k = a.log2T, q = a.tail_p - 1;
+      for (int j = tid; j < r; j += kRQThreads) {
+        const int ap = j >> k, bp = j & ((1 << k) - 1);
+        long long S = 0;
+        for (int aa = 0; aa < a.tail_p; ++aa) {
+          const long long z = tz[(aa << k) + bp];
+          int h;
+          if (aa == ap || aa == 0)
+            h = 1;
+          else if (ap == 0)
+            h = -1;
+          else
+            h = chi[(ap - aa + q) % q];
+          S += h > 0 ? z : -z;
+        }
+        const float yv = fixed_times_const(S, a.tail_j, a.t_hi, a.t_lo);
+        lmax = fmaxf(lmax, fabsf(yv));
+        sy[tail_start + j] = yv;
       }
     }
     sync();

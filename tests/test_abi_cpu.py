@@ -59,7 +59,11 @@ def test_argument_checks_need_no_gpu(lib):
     assert b"bits" in lib.dptq_last_error_message()
     # K not a multiple of 32 / bad Hadamard layout / null pointers / sizes
     assert lib.dptq_rotate_quant_act(dummy, 4, 100, 64, 4, dummy, dummy, None) == 2
-    assert lib.dptq_rotate_quant_act(dummy, 4, 1536 + 96, 512, 4, dummy, dummy, None) == 2
+    # a tail of 96 = 12 x 8 has a Paley factor (11 is prime): the shape checks pass
+    assert lib.dptq_rotate_quant_act(dummy, 4, 1536 + 96, 512, 4, dummy, dummy, None) != 2
+    # a tail of 736 = 23 x 32 has none of order at most 256 (91, 183 composite; 368 too large)
+    assert lib.dptq_rotate_quant_act(dummy, 4, 1024 + 736, 1024, 4, dummy, dummy, None) == 2
+    assert b"Paley" in lib.dptq_last_error_message()
     assert lib.dptq_rotate_quant_act(None, 4, 256, 256, 4, dummy, dummy, None) == 1
     assert lib.dptq_rotate_quant_act(dummy, -1, 256, 256, 4, dummy, dummy, None) == 1
     assert lib.dptq_rotate_quant_act(dummy, 0, 256, 256, 4, dummy, dummy, None) == 0   # M == 0: no-op

@@ -468,3 +468,48 @@ def test_concatenated_group_handles(dp, orc, wl_name, group, M, bits):
     hot = [t for t in range(M) if np.abs(x[t].astype(np.float32)).max() > 50]
     rows = None if M <= 64 else sample(M, 16, 11, must=hot[:4])
     check_qlinear(dp, orc, x, W, B, bits, rows=rows, cols=tile_sample(W.shape[0], 12))
+
+
+# ----------------------------------------------------------------------------- non-power-of-two tails
+# K = 11008 with blocks of 4096 leaves a tail of 2816 = 44 x 64 (LLaMA-2-7B's down input),
+# K = 13824 leaves 1536 = 12 x 128 (LLaMA-2-13B's), 448 = 256 + 12 x 16: the tail block's
+# Hadamard matrix is Paley's H_p (x) the Sylvester H_(2^k) (Section 2 Eq. 4, R^T R = I).
+PALEY_CASES = [(11008, 4096, 4), (13824, 4096, 3), (256 + 192, 256, 6)]
+
+
+@pytest.mark.parametrize("K,B,M", PALEY_CASES)
+def test_paley_tail_rotation_and_codes(dp, orc, K, B, M):
+    assert orc.tail_factor(K % B)[0] > 1
+    wl = inputs.llama2_7b_decode()
+    x = np.concatenate([inputs.activations(wl, M, K), edge_rows(K)])
+    y_ref = orc.rotate(x, B)
+    parity.check_rotation(gpu_rotate(dp, x, B), y_ref)
+    for bits in (4, 8):
+        c_ref, s_ref = orc.rotate_quant_act(x, B, bits)
+        c, s = gpu_codes(dp, x, B, bits, orc)
+        parity.check_scales(s, s_ref)
+        parity.check_codes(c, c_ref, y_ref, s_ref, bits)
+
+
+@pytest.mark.parametrize("K,B", [(11008, 4096), (448, 256)])
+def test_paley_tail_pack_and_qlinear(dp, orc, K, B):
+    """Weight packing folds the same R (Eq. 5), and the qlinear layer (two launches: the
+    fused decode launch takes power-of-two tails only) matches the oracle, at 8 tokens
+    and at 130; the oracle's dense fp64 rotation costs about 0.3 s per row at K = 11008,
+    so it checks sampled rows and one channel per weight tile."""
+    N = 384
+    W = inputs.weights(N, K, layer=6, proj=6)
+    cols = tile_sample(N, 13)
+    q_ref, sw_ref = orc.pack_weights(np.ascontiguousarray(W[cols]), B)
+    layer = dp.dptq_pack_weights(torch.from_numpy(W).to(DEV), B)
+    wq, sw = dp.dptq_get_packed(layer)
+    parity.check_scales(sw[cols], sw_ref)
+    parity.check_codes(orc.unpack_nibbles(wq[cols], K), q_ref, orc.rotate(np.ascontiguousarray(W[cols]), B),
+                       sw_ref, 4)
+    layer.close()
+    wl = inputs.llama2_7b_decode()
+    for M in (8, 130):
+        x = inputs.activations(wl, M, K)
+        rows = sample(M, 6, M, must=(127, 128))
+        for bits in (4, 8):
+            check_qlinear(dp, orc, x, W, B, bits, rows=rows, cols=cols)

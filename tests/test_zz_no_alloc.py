@@ -99,5 +99,13 @@ def test_static_scratch_rejects_shapes_beyond_its_limit(dp):
     out2 = torch.empty((4, 128), dtype=torch.float16, device="cuda")
     st, msg = _static_call(dp, layer2, x2, 4, out2)
     assert st == 2 and "16384" in msg
+    # a Paley tail block (K = 1024 + 96 = 12 x 8): served by dptq_qlinear, not here
+    W3 = torch.from_numpy(inputs.weights(128, 1120)).cuda()
+    layer3 = dp.dptq_pack_weights(W3, 1024)
+    x3 = torch.zeros((4, 1120), dtype=torch.float16, device="cuda")
+    out3 = torch.empty((4, 128), dtype=torch.float16, device="cuda")
+    st, msg = _static_call(dp, layer3, x3, 4, out3)
+    assert st == 2 and "tail" in msg
     layer.close()
     layer2.close()
+    layer3.close()
