@@ -660,7 +660,20 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
     // ------------------------------------------------------------ epilogue
     pdl_wait();   // scales come from the previous kernel; `out` may still be read by it
     bool epi_ok = true;
-    if constexpr (FUSED) epi_ok = mbar_wait(aready, 0, abort_flag, a.err, kDevTimeoutGrid, a.wait_cycles);
+    if constexpr (FUSED) {
+      epi_ok = mbar_wait(aready, 0, abort_flag, a.err, kDevTimeoutGrid, a.wait_cycles);
+      // This CTA's producer has passed its wait on the row counter (or gave up): the last
+      // CTA to get here resets both grid counters for the next launch, which touches them
+      // only after this grid ends.  Done here, while the weights still stream, the atomic's
+      // round trip stays off the kernel's exit.
+      if (threadIdx.x == kEpiWarp0 * 32) {
+        const uint32_t prev = atom_add_acq_rel_gpu(a.gsync + 1, 1u);
+        if (prev == gridDim.x - 1) {
+          a.gsync[0] = 0u;
+          a.gsync[1] = 0u;
+        }
+      }
+    }
     const float* __restrict__ sa_g = a.sa;
     const float* __restrict__ sw_g = a.sw;
     __half* __restrict__ out_g = a.out;
@@ -880,34 +893,54 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
           DPTQ_TRACE_POINT(tr, 5);
         }
         if (!epi_sync()) break;
-        if (flag[1]) {
+        if (flag[1] && f32) {
+          // The slot holds the whole tile.  Chunks of 16 tokens, the next chunk's reads
+          // issued before the current chunk is written, so that one L2 round trip covers
+          // two chunks.
+          float4 p0[4], p1[4];
+          auto load_slot = [&](int c, float4 (&d)[4]) {
+#pragma unroll
+            for (int j = 0; j < 4; ++j) d[j] = __ldcg(reinterpret_cast<const float4*>(wslf + (c / 4 + j) * 512));
+          };
+          auto emit = [&](int c, const float4 (&d)[4]) {
+            float vf[16];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+              vf[4 * j] = d[j].x * 512.f;   // exact: one segment's sums are below 2^24 units
+              vf[4 * j + 1] = d[j].y * 512.f;
+              vf[4 * j + 2] = d[j].z * 512.f;
+              vf[4 * j + 3] = d[j].w * 512.f;
+            }
+#pragma unroll
+            for (int j = 0; j < 4; ++j)   // zero for the next launch
+              __stcg(reinterpret_cast<float4*>(wslf + (c / 4 + j) * 512), make_float4(0.f, 0.f, 0.f, 0.f));
+            write_out(c, vf, nullptr);
+          };
+          load_slot(0, p0);
+#pragma unroll 1
+          for (int c0 = 0; c0 < NT; c0 += 32) {
+            if (NT > 64) sa_grp = sa_group(c0);
+            const bool two = c0 + 16 < NT;
+            if (two) load_slot(c0 + 16, p1);
+            emit(c0, p0);
+            if (two) {
+              if (c0 + 32 < NT) load_slot(c0 + 32, p0);
+              emit(c0 + 16, p1);
+            }
+          }
+        } else if (flag[1]) {
 #pragma unroll 1
           for (int c0 = 0; c0 < NT; c0 += 16) {
             if (NT > 64 && (c0 & 31) == 0) sa_grp = sa_group(c0);
             float vf[16];
-            if (f32) {
+            int v[16];
 #pragma unroll
-              for (int j = 0; j < 4; ++j) {
-                const float4 t = __ldcg(reinterpret_cast<const float4*>(wslf + (c0 / 4 + j) * 512));
-                vf[4 * j] = t.x * 512.f;   // exact: one segment's sums are below 2^24 units
-                vf[4 * j + 1] = t.y * 512.f;
-                vf[4 * j + 2] = t.z * 512.f;
-                vf[4 * j + 3] = t.w * 512.f;
-              }
+            for (int i = 0; i < 16; ++i) v[i] = __ldcg(wsl + (c0 + i) * 128 + q * 32 + lane);
 #pragma unroll
-              for (int j = 0; j < 4; ++j)
-                __stcg(reinterpret_cast<float4*>(wslf + (c0 / 4 + j) * 512), make_float4(0.f, 0.f, 0.f, 0.f));
-              write_out(c0, vf, nullptr);
-            } else {
-              int v[16];
+            for (int i = 0; i < 16; ++i) __stcg(wsl + (c0 + i) * 128 + q * 32 + lane, 0);
 #pragma unroll
-              for (int i = 0; i < 16; ++i) v[i] = __ldcg(wsl + (c0 + i) * 128 + q * 32 + lane);
-#pragma unroll
-              for (int i = 0; i < 16; ++i) __stcg(wsl + (c0 + i) * 128 + q * 32 + lane, 0);
-#pragma unroll
-              for (int i = 0; i < 16; ++i) vf[i] = __int2float_rn(v[i]);
-              write_out(c0, vf, v);
-            }
+            for (int i = 0; i < 16; ++i) vf[i] = __int2float_rn(v[i]);
+            write_out(c0, vf, v);
           }
         }
         if (etid == 0) {
@@ -926,17 +959,6 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem_base, a.tmem_cols);
-  }
-  if constexpr (FUSED) {
-    // Every producer has passed its wait on the row counter: the last CTA out resets
-    // both counters for the next launch (which reads them only after this grid ends).
-    if (threadIdx.x == 0) {
-      const uint32_t prev = atom_add_acq_rel_gpu(a.gsync + 1, 1u);
-      if (prev == gridDim.x - 1) {
-        a.gsync[0] = 0u;
-        a.gsync[1] = 0u;
-      }
-    }
   }
   if (threadIdx.x == 0) DPTQ_TRACE_POINT(tr, 120);
 }
