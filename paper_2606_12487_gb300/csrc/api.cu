@@ -166,8 +166,12 @@ struct Scratch {
   float* sa = nullptr;
   size_t sa_count = 0;
   int32_t* ws = nullptr;
-  uint32_t* counters = nullptr;   // [num_sms] split-tile arrivals, then [2] fused-launch grid counters
+  // [SMs] split-tile arrivals, [2] fused-launch grid counters, then (128-byte aligned)
+  // the row-maximum slots of the fused launch's row parts, [64][kRowMaxStride]
+  uint32_t* counters = nullptr;
+  size_t counter_words = 0;
   uint32_t* gsync = nullptr;
+  uint32_t* pmax = nullptr;
   int* err = nullptr;
   int num_sms = 0;
   std::vector<std::pair<void*, size_t>> retired;   // superseded act / sa buffers, still allocated
@@ -182,9 +186,13 @@ bool capturing(cudaStream_t s) {
 }
 
 constexpr int kMaxNT = 256;
-// Rows of up to 4 chunks of 4096 take the fused launch (its rotation runs each row's
-// butterflies twice when the row has more than one chunk).
+// Rows of up to 16384 elements take the fused launch (each of a row's four parts rotates
+// at most 4096 of them).
 constexpr int kFusedMaxKPad = 16384;
+// Counter words: split-tile arrivals and grid counters, then the row-maximum slots, one
+// 128-byte line per row (only the parts of one row poll a line).
+size_t pmax_offset(int sms) { return ((size_t)sms + 2 + 31) & ~(size_t)31; }
+size_t counter_words(int sms) { return pmax_offset(sms) + (size_t)64 * kRowMaxStride; }
 
 // Every device allocation of the library goes through here.  Host-side fault injection
 // for tests of the out-of-memory path: with DPTQ_FAULT_ALLOC=n (n >= 1) in the
@@ -221,10 +229,10 @@ dptq_status ensure_scratch(int dev, size_t act_bytes, size_t sa_count, cudaStrea
     uint32_t* counters = nullptr;
     int* err = nullptr;
     cudaError_t e = dev_malloc(reinterpret_cast<void**>(&ws), ws_bytes);
-    if (e == cudaSuccess) e = dev_malloc(reinterpret_cast<void**>(&counters), sizeof(uint32_t) * (sms + 2));
+    if (e == cudaSuccess) e = dev_malloc(reinterpret_cast<void**>(&counters), sizeof(uint32_t) * counter_words(sms));
     if (e == cudaSuccess) e = dev_malloc(reinterpret_cast<void**>(&err), sizeof(int));
     if (e == cudaSuccess) e = cudaMemset(ws, 0, ws_bytes);
-    if (e == cudaSuccess) e = cudaMemset(counters, 0, sizeof(uint32_t) * (sms + 2));
+    if (e == cudaSuccess) e = cudaMemset(counters, 0, sizeof(uint32_t) * counter_words(sms));
     if (e == cudaSuccess) e = cudaMemset(err, 0, sizeof(int));
     if (e != cudaSuccess) {   // nothing has used these yet: release them and stay uninitialized
       if (ws) cudaFree(ws);
@@ -232,6 +240,8 @@ dptq_status ensure_scratch(int dev, size_t act_bytes, size_t sa_count, cudaStrea
       if (err) cudaFree(err);
       return cuda_fail(e, "scratch allocation");
     }
+    sc.counter_words = counter_words(sms);
+    sc.pmax = counters + pmax_offset(sms);
     // DPTQ_MAX_GRID=n caps the CTAs of a GEMM launch (tuning experiments; default: the
     // device's SMs).
     if (const char* v = std::getenv("DPTQ_MAX_GRID")) {
@@ -294,7 +304,10 @@ dptq_status run_gemm(dptq_handle h, const GemmPlan& plan0, const uint8_t* act, c
   g.gsync = sc->gsync;
   g.err = sc->err;
   g.wait_cycles = wait_cycles_setting();
-  if (plan.fused) g.rq_shortfall = take_rows_shortfall();
+  if (plan.fused) {
+    g.rq_shortfall = take_rows_shortfall();
+    g.pre_stages = pre_stages_setting();
+  }
   DPTQ_CUDA(launch_gemm(plan, s, true), "qgemm launch");
   return DPTQ_OK;
 }
@@ -324,6 +337,17 @@ bool l2_prefetch_allowed() {
     return !(v && v[0] == '0');
   }();
   return on;
+}
+
+// Weight stages a fused launch requests before its token rows are ready (DPTQ_PRE_STAGES,
+// a tuning knob; default 2).
+int pre_stages_setting() {
+  static const int v = [] {
+    const char* e = std::getenv("DPTQ_PRE_STAGES");
+    const int n = e ? std::atoi(e) : 2;
+    return n < 1 ? 1 : n;
+  }();
+  return v;
 }
 
 long long wait_cycles_setting() {
@@ -570,11 +594,14 @@ dptq_status dptq_qlinear(dptq_handle h, const void* x_fp16, int M, int bits, voi
   // Small M: one launch that rotates and quantizes the rows and runs the GEMM.
   GemmPlan fp;
   if (fused_allowed() && h->K_pad <= kFusedMaxKPad && pow2_tail(h->K, h->had_block) &&
-      plan_gemm(M, h->N, h->K_pad, bits, sc->num_sms, fp, kRQPartSmemBytes) && fp.M_pad == plan.M_pad) {
+      plan_gemm(M, h->N, h->K_pad, bits, sc->num_sms, fp, kRQPartSmemBytes) && fp.M_pad == plan.M_pad &&
+      fp.M_pad <= 64 && fused_rotation_variant(h->K, h->had_block, h->K % h->had_block, fp.args.rq_np) >= 0) {
     int nfull, tail, log2B;
     if ((st = check_shape(h->K, h->had_block, nfull, tail, log2B)) != DPTQ_OK) return st;
     fp.args.rq = make_rq(x_fp16, M, fp.M_pad, h->K, h->KB, h->had_block, nfull, tail, log2B, bits, sc->sa, sc->act);
     fp.args.rq.signs = h->signs;
+    fp.args.rq.np = fp.args.rq_np;
+    fp.args.rq.pmax = sc->pmax;
     return run_gemm(h, fp, sc->act, sc->sa, out_fp16, nullptr, sc, s);
   }
   if ((st = quantize_into_scratch(h, x_fp16, M, bits, plan, sc, s)) != DPTQ_OK) return st;
@@ -756,11 +783,11 @@ dptq_status dptq_last_device_error(dptq_handle h) {
       DPTQ_CUDA(cudaMemcpy(&word, sc.err, sizeof(int), cudaMemcpyDeviceToHost), "cudaMemcpy(err)");
       if (word != 0) {
         // A wait gave up: clear the word, the split-tile sums and every counter (split-tile
-        // arrivals and the fused launch's two grid counters) the aborted kernel may have
-        // left non-zero.
+        // arrivals, the fused launch's two grid counters and its row-maximum slots) the
+        // aborted kernel may have left non-zero.
         DPTQ_CUDA(cudaMemset(sc.err, 0, sizeof(int)), "cudaMemset(err)");
         DPTQ_CUDA(cudaMemset(sc.ws, 0, (size_t)sc.num_sms * kMaxNT * 128 * sizeof(int32_t)), "cudaMemset(ws)");
-        DPTQ_CUDA(cudaMemset(sc.counters, 0, sizeof(uint32_t) * (sc.num_sms + 2)), "cudaMemset(counters)");
+        DPTQ_CUDA(cudaMemset(sc.counters, 0, sizeof(uint32_t) * sc.counter_words), "cudaMemset(counters)");
       }
     }
   }

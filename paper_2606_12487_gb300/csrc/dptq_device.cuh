@@ -76,6 +76,7 @@ enum DeviceError : int {
   kDevTimeoutTmemEmpty = 0x105,
   kDevTimeoutDrain = 0x106,
   kDevTimeoutGrid = 0x107,     // grid-wide phase barrier did not complete
+  kDevTimeoutRowMax = 0x108,   // a row's parts did not all post their maxima
 };
 
 // About one second at the GB300's ~2 GHz SM clock: any single wait longer than this

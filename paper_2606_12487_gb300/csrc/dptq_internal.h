@@ -37,6 +37,8 @@ enum RQMode : int {
   kRQWeights = 3,  // packed sign-magnitude int4 weight tiles + per-channel scales
 };
 
+constexpr int kRowMaxStride = 32;   // words per row of the fused launch's row-maximum slots
+
 struct RQArgs {
   const __half* x;   // [rows_in][K] binary16, row-major
   const int8_t* signs;  // randomized Hadamard diagonal [K] (+1 / -1, 16-byte aligned) or null
@@ -59,6 +61,11 @@ struct RQArgs {
   int tail_j;
   float t_hi, t_lo;
   int bits;          // 4 or 8
+  // Fused decode launch: parts per row and the row-maximum slots, kRowMaxStride words
+  // per row of which the first np are used (1 + the bits of each part's largest |y|;
+  // 0 = not yet written; zero between launches).
+  int np;
+  uint32_t* pmax;
   float* scales;     // [rows_out] (rows >= rows_in get 0); may be null in kRQY
   void* out;         // mode-dependent destination
 };
@@ -127,6 +134,11 @@ struct GemmArgs {
   uint32_t tmem_cols;
   int out_vec;         // `out` is 16-byte aligned: the epilogue stores 8 channels at a time
   long long l2_prefetch;  // weight bytes past the first ring stages each CTA requests into L2 up front (0: none)
+  // Fused launch: weight stages the producer requests before the token rows are ready;
+  // the rest of the ring and the L2 prefetch wait for the rows (while the rows are
+  // rotated, the parts' exchanges of their maxima cross the memory system, and a full
+  // ring fill in flight delays them by microseconds).
+  int pre_stages;
   // Fused decode launches only: the rotation + quantization of the M_pad token rows
   // (written to `act` / `sa` by the converter warps of CTAs 0, 1, ...) and the two grid
   // counters [rows ready, CTAs done] that order it before the GEMM (zero between launches).
@@ -154,6 +166,9 @@ struct GemmPlan {
 // `rot_smem` > 0 plans the fused decode kernel: that many extra bytes of shared memory
 // for the rotation of one row, two k-blocks per stage; false if it does not fit.
 bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan, int rot_smem = 0);
+// Row split of the fused launch for K, B, the (power-of-two) tail and np parts per row:
+// kPartBlocks, kPartSlice4 or kPartSlice8 (rotate_row.cuh), or -1 when none applies.
+int fused_rotation_variant(int K, int B, int tail, int np);
 cudaError_t launch_gemm(const GemmPlan& plan, cudaStream_t s, bool pdl);
 
 // Programmatic dependent launch is on unless the environment sets DPTQ_PDL=0 (kernels
@@ -170,6 +185,7 @@ long long wait_cycles_setting();
 int take_rows_shortfall();
 // Decode GEMM launches prefetch their weight share into L2 unless DPTQ_L2PF=0.
 bool l2_prefetch_allowed();
+int pre_stages_setting();
 // The GEMM operand rows are rotated and quantized by the whole-row kernel (sums kept in
 // registers) unless DPTQ_ROWS_KERNEL=0 (the per-row kernel with an fp32 row in shared
 // memory).

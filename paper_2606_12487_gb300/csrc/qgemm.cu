@@ -170,12 +170,14 @@ struct Smem {
 };
 
 // RQV != 0 (decode, two-block stages) makes the launch FUSED: it first rotates and
-// quantizes the token rows itself.  Each row is split into rq_np parts (RQV = 16 / rq_np
-// values per chunk and thread: 4 with four parts, 8 with two), and the converter warps
-// of CTA c handle the (row, part) items c, c + G, ... and publish them on a grid counter;
-// every producer streams its first weight stages meanwhile and requests activation tiles
-// once all items are in; the epilogue reads the token scales after the same point.  The
-// last CTA to finish resets the counters.
+// quantizes the token rows itself.  Each row is split into rq_np parts, each part
+// rotating only its own outputs (RQV = kPartBlocks: whole blocks per part;
+// kPartSlice4 / kPartSlice8: slices of one block, 4 or 8 values per thread); the parts
+// of a row exchange their maxima through global slots, and the converter warps publish
+// the rows on a grid counter.  Every producer streams its first weight stages meanwhile
+// and requests activation tiles once all rows are in; the epilogue reads the token
+// scales after the same point, and the last CTA to get there resets the counters and
+// the slots.
 template <int NT, int KPS, int RQV>
 __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a) {
   constexpr bool FUSED = RQV != 0;
@@ -348,6 +350,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
         const int s = rg.s;
         const bool tg = kTraceStages > 10 && wprod && leader && g >= 8 && g < 11;   // clocked stages (trace builds)
         (void)tg;
+        if (FUSED && wprod && g == a.pre_stages &&
+            !mbar_wait_warp(aready, 0, abort_flag, a.err, kDevTimeoutGrid, a.wait_cycles)) {
+          ok = false;   // the rows never became ready
+          break;
+        }
         if (tg) DPTQ_TRACE_CLOCK(tr, 224 + 3 * (g - 8));
         if (!mbar_wait_warp(&empty[s], rg.ph ^ 1u, abort_flag, a.err, kDevTimeoutEmpty, a.wait_cycles)) {
           ok = false;
@@ -490,23 +497,30 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
     // ------------------------------------------------------------ converters
     const int ctid = threadIdx.x - kConvWarp0 * 32;   // 0..255
     if constexpr (FUSED) {
-      // Rotate + quantize work items c, c + G, ... (item = row * rq_np + part) into the
-      // activation planes and scales, then publish them.  The 8 converter warps meet
-      // at named barrier 1.
+      // Rotate + quantize this CTA's (row, part) items into the activation planes and
+      // scales, then publish them.  The 8 converter warps meet at named barrier 1.
       pdl_wait();   // the rows come from the previous kernel
       if (ctid == 0) {
         DPTQ_TRACE_POINT(tr, 125);
         DPTQ_TRACE_CLOCK(tr, 160);
       }
       const auto csync = [] { asm volatile("bar.sync 1, %0;" ::"n"(kConvThreads) : "memory"); };
+      // Rows go out in rounds of G / np rows, CTA c taking part c % np of rows
+      // c / np, c / np + G / np, ...: the parts of a row, which wait for one another's
+      // maxima, always run in the same round.
+      const int np = a.rq.np;
+      const int rpr = (int)gridDim.x / np;
       int nitems = 0;
-      for (int item = blockIdx.x; item < a.rq_items; item += gridDim.x) {
-        if (nitems) csync();   // the previous item's readers are done with the scratch
-        // Four parts: rows of up to four 4096-element chunks; two parts: up to two.
-        constexpr int kMaxChunks = RQV == 4 ? 4 : 2;
-        rotate_quant_row_part_fast<RQV == 4 ? 4 : 8, kMaxChunks>(a.rq, item / a.rq_np, item % a.rq_np, rot_smem,
-                                                                 ctid, csync);
-        ++nitems;
+      if ((int)blockIdx.x < rpr * np) {
+        const int part = (int)blockIdx.x % np;
+        for (int row = (int)blockIdx.x / np; row < a.rq.rows_out; row += rpr) {
+          if (nitems) csync();   // the previous row's readers are done with the scratch
+          if constexpr (RQV == kPartBlocks)
+            rotate_quant_part_blocks(a.rq, row, part, rot_smem, ctid, csync, a.wait_cycles, a.err);
+          else
+            rotate_quant_part_slice<RQV>(a.rq, row, part, rot_smem, ctid, csync, a.wait_cycles, a.err);
+          ++nitems;
+        }
       }
       if (ctid == 0) {
         DPTQ_TRACE_POINT(tr, 126);
@@ -668,9 +682,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
       // round trip stays off the kernel's exit.
       if (threadIdx.x == kEpiWarp0 * 32) {
         const uint32_t prev = atom_add_acq_rel_gpu(a.gsync + 1, 1u);
-        if (prev == gridDim.x - 1) {
+        if (prev == gridDim.x - 1) {   // every part has also read its row's maxima
           a.gsync[0] = 0u;
           a.gsync[1] = 0u;
+          for (int r = 0; r < a.rq.rows_out; ++r)
+            *reinterpret_cast<uint4*>(a.rq.pmax + kRowMaxStride * r) = make_uint4(0u, 0u, 0u, 0u);
         }
       }
     }
@@ -1096,11 +1112,11 @@ bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan, i
   a.l2_prefetch = (nt <= 64 && m_tiles == 1 && l2_prefetch_allowed()) ? 512LL * 1024 : 0;
   a.rq = RQArgs{};
   a.gsync = nullptr;
-  // Fused: every token row is split into 4 parts (each quantizes and writes a quarter of
-  // it) when each part gets a CTA of its own; else into 2 parts with a CTA each, for rows
-  // of at most two 4096-element chunks; else into 4 parts with at most two per CTA.  A
-  // launch whose grid is smaller than that leaves the rows to the separate
-  // rotate-quantize launch (no fused plan).
+  // Fused: every token row is split into 4 parts (each rotates and quantizes its share
+  // of the row) when each part gets a CTA of its own; else into 2 parts with a CTA each,
+  // for rows of at most 8192 elements (at most 4096 per part); else into 4 parts in two
+  // rounds of rows.  A launch whose grid is smaller than that leaves the rows to the
+  // separate rotate-quantize launch (no fused plan).
   int np = 1;
   if (fused) {
     if ((long long)M_pad * 4 <= G)
@@ -1115,8 +1131,25 @@ bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan, i
   a.rq_np = np;
   a.rq_items = fused ? M_pad * np : 0;
   a.rq_shortfall = 0;
+  a.pre_stages = 2;
   a.wait_cycles = kWaitTimeoutCycles;
   return true;
+}
+
+// How the fused launch splits a row over its np parts (two or four): slices of one
+// block when the row has fewer blocks than parts (K a multiple of B, n = np B / K >= 2
+// parts per block, slices of 1024 or 2048 elements), else whole blocks (every part at
+// most 4096 elements: K <= 4096 np).  -1: neither applies.
+int fused_rotation_variant(int K, int B, int tail, int np) {
+  if (np != 2 && np != 4) return -1;
+  if (tail == 0 && K % B == 0 && (np * B) % K == 0) {
+    const int n = np * B / K;
+    if (n >= 2 && B / n == 1024) return kPartSlice4;
+    if (n >= 2 && B / n == 2048) return kPartSlice8;
+  }
+  const int gr = B > 128 ? B : 128;
+  const int ng = (K + gr - 1) / gr;
+  return (ng + np - 1) / np * gr <= 4096 ? kPartBlocks : -1;
 }
 
 template <int NT, int KPS, int RQV = 0>
@@ -1138,14 +1171,20 @@ static cudaError_t launch_nt(const GemmPlan& plan, cudaStream_t s, bool pdl) {
 
 cudaError_t launch_gemm(const GemmPlan& plan, cudaStream_t s, bool pdl) {
   if (plan.fused) {
-    const bool four = plan.args.rq_np == 4;
-    if (!four && plan.args.rq_np != 2) return cudaErrorInvalidValue;
+    const int v = fused_rotation_variant(plan.args.rq.K, plan.args.rq.B, plan.args.rq.tail, plan.args.rq_np);
+    if (v < 0 || plan.args.rq.np != plan.args.rq_np) return cudaErrorInvalidValue;
+#define DPTQ_FUSED_NT(nt)                                                      \
+  case nt:                                                                     \
+    return v == kPartSlice4   ? launch_nt<nt, 2, kPartSlice4>(plan, s, pdl)    \
+           : v == kPartSlice8 ? launch_nt<nt, 2, kPartSlice8>(plan, s, pdl)    \
+                              : launch_nt<nt, 2, kPartBlocks>(plan, s, pdl);
     switch (plan.nt) {
-      case 16: return four ? launch_nt<16, 2, 4>(plan, s, pdl) : launch_nt<16, 2, 8>(plan, s, pdl);
-      case 32: return four ? launch_nt<32, 2, 4>(plan, s, pdl) : launch_nt<32, 2, 8>(plan, s, pdl);
-      case 64: return four ? launch_nt<64, 2, 4>(plan, s, pdl) : launch_nt<64, 2, 8>(plan, s, pdl);
+      DPTQ_FUSED_NT(16)
+      DPTQ_FUSED_NT(32)
+      DPTQ_FUSED_NT(64)
       default: return cudaErrorInvalidValue;
     }
+#undef DPTQ_FUSED_NT
   }
   if (plan.kps == 2) {
     switch (plan.nt) {

@@ -734,211 +734,404 @@ __device__ __forceinline__ uint32_t e4m3_byte(float v) { return e4m3x2(v, 0.f) &
 
 static_assert(kRQPartSmemBytes == kChunkPadded * 8 + 2 * kChunk + 16 * 8, "part scratch layout");
 
-// The share `part` of 16 / VPC parts of one row in the fused decode launch, for rows of
-// at most MAXCH chunks (K <= 4096 MAXCH; VPC * MAXCH <= 16): the codes and scale of
-// rotate_quant_row<kRQAct>, computed for low latency rather than throughput.  This code
-// runs once per launch, so its instructions are fetched cold; it is kept small (rolled
-// chunk loop, one butterfly body for all rounds) so that repeated work runs from the
-// instruction cache.
-//   * The next chunk's 32 bytes per thread are requested before the current chunk's
-//     butterflies run, so the row's global loads overlap the arithmetic.
-//   * The VPC values of each chunk that this part quantizes are converted to fp32 as the
-//     chunk finishes and stay in registers (at most 16), so no butterflies are redone.
-//   * The row absmax: each thread converts its largest |S| of each block size once (the
-//     conversion is odd and monotone, so the fp32 of the largest |S| is the largest |y|);
-//     the warp maximum is one redux on the fp32 bit patterns (non-negative floats order as
-//     their bits), then one shared-memory step across the 8 warps.
-//   * All of the part's codes are staged in shared memory (the transpose buffer, free once
-//     the butterflies are done) and stored after one barrier, as 32-bit words whose four
-//     codes are consecutive in k.
+// ---- one row's rotation split over the parts of the fused decode launch
+// Each of the np parts of a row rotates only its own outputs, so the parts share the
+// work instead of repeating it; the row absmax, which every code depends on, is then
+// exchanged between the parts through one slot per part in global memory.
+//   * Whole blocks (kPartBlocks): the row splits into np ranges of whole 128-aligned
+//     granules (a granule is max(B, 128) elements: whole Hadamard blocks), each at most
+//     4096 elements, rotated like one chunk of rotate_quant_row.
+//   * Block slices (kPartSlice4 / kPartSlice8): when a row has fewer blocks than parts,
+//     each block of B = n L elements is shared by n parts.  With Sylvester's ordering
+//     H_B = H_n (x) H_L, so output slice p' of the block is H_L applied to
+//     v = sum_a H_n[p'][a] x_a, x_a the a-th L-element slice of the block's input: a part
+//     combines the n input slices at its L positions (exact) and runs the L-point
+//     butterflies, L = 256 V (V = 4 or 8 values per thread).
+enum : int { kPartBlocks = 1, kPartSlice4 = 4, kPartSlice8 = 8 };
+
+// Granule range [g0, g1) of `part` when ng granules are split over np parts.
+__device__ __forceinline__ void part_granules(int ng, int np, int part, int& g0, int& g1) {
+  g0 = part * ng / np;
+  g1 = (part + 1) * ng / np;
+}
+
+// Row absmax over the parts.  Thread 0 of the part stores 1 + the bits of its own
+// maximum (non-negative floats order as their bit patterns; 0 marks an empty slot) in
+// slot [row][part] (one 128-byte line per row), then reads the row's first four slots,
+// pausing between reads so that the pollers of a line leave the store of the last part
+// a way in, until the first np are set; the
+// slots are cleared for the next launch once every part of the launch is past this
+// point.  A slot holds only its own value, so relaxed accesses suffice.  Bounded: on
+// timeout the error word is set and the part's own maximum stands in.
+__device__ __forceinline__ float part_absmax_exchange(uint32_t* slots, int np, int part, float mine,
+                                                      long long wait_cycles, int* err) {
+  asm volatile("st.relaxed.gpu.global.u32 [%0], %1;" ::"l"(slots + part), "r"(__float_as_uint(mine) + 1u) : "memory");
+  const long long t0 = clock64();
+  while (true) {
+    uint32_t v[4];
+    asm volatile("ld.relaxed.gpu.global.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3])
+                 : "l"(slots)
+                 : "memory");
+    bool all = true;
+    uint32_t m = 0u;
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+      if (i < np) {
+        all = all && v[i] != 0u;
+        m = v[i] > m ? v[i] : m;
+      }
+    if (all) return __uint_as_float(m - 1u);
+    if (clock64() - t0 > wait_cycles) {
+      atomicCAS(err, 0, (int)kDevTimeoutRowMax);
+      return mine;
+    }
+    __nanosleep(100);
+  }
+}
+
+// The part's largest |y| from the fp32 of each thread's largest |y| (`tmax`, >= 0): one
+// redux per warp on the bit patterns, the 8 warp maxima through `redf`, then the
+// exchange between the parts (thread 0) and its broadcast.  Two barriers.
+template <class Sync>
+__device__ __forceinline__ float part_row_absmax(const RQArgs& a, int row, int part, float tmax, float* redf, int tid,
+                                                 Sync sync, long long wait_cycles, int* err) {
+  const uint32_t wmax = __reduce_max_sync(0xffffffffu, __float_as_uint(tmax));
+  if ((tid & 31) == 0) redf[tid >> 5] = __uint_as_float(wmax);
+  sync();
+  if (tid == 0) {
+    float pm = redf[0];
+#pragma unroll
+    for (int w = 1; w < kRQThreads / 32; ++w) pm = fmaxf(pm, redf[w]);
+    redf[8] = part_absmax_exchange(a.pmax + kRowMaxStride * row, a.np, part, pm, wait_cycles, err);
+  }
+  sync();
+  return redf[8];
+}
+
+// Codes k .. k + 3 of `row` (k % 4 == 0) into the GEMM operand planes (the 128-byte
+// swizzled K-major layout of rotate_quant_row<kRQAct>).
+__device__ __forceinline__ void part_store4(const RQArgs& a, int row, int k, uint32_t w0, uint32_t w1) {
+  uint8_t* act = static_cast<uint8_t*>(a.out);
+  const int kb = k >> 7, j = (k >> 4) & 7;
+  const size_t off = ((size_t)kb * a.rows_out + row) * 128 + ((j ^ (row & 7)) << 4) + (k & 15);
+  *reinterpret_cast<uint32_t*>(act + off) = w0;
+  if (a.bits == 8) *reinterpret_cast<uint32_t*>(act + (size_t)a.KB * a.rows_out * 128 + off) = w1;
+}
+
+// Padding row (row >= rows_in): zero codes, the K_pad / 4 words split evenly over the
+// parts, and a zero scale.
+__device__ __forceinline__ void part_zero_row(const RQArgs& a, int row, int part, int tid) {
+  const int W = a.KB * 32;
+  for (int w = W * part / a.np + tid; w < W * (part + 1) / a.np; w += kRQThreads) part_store4(a, row, 4 * w, 0u, 0u);
+  if (part == 0 && tid == 0 && a.scales != nullptr) a.scales[row] = 0.f;
+}
+
+// Staged E4M3 byte(s) of one code: plane 0 (A4, or the A8 hi part) and plane 1 (A8 lo).
+__device__ __forceinline__ void part_code_bytes(float q, int bits, uint32_t& b0, uint32_t& b1) {
+  if (bits == 4) {
+    b0 = e4m3_byte(q);
+    b1 = 0u;
+  } else {
+    const float m = fabsf(q);
+    const float h = __fmul_rn(floorf(__fmul_rn(m, 0.0625f)), 16.f);
+    b0 = e4m3_byte(__fadd_rn(copysignf(h, q), 0.0f));   // + 0: no negative zeros
+    b1 = e4m3_byte(__fadd_rn(copysignf(__fsub_rn(m, h), q), 0.0f));
+  }
+}
+
+// Whole blocks: this part's granules [c0, c0 + len) of the row (len <= 4096), rotated as
+// one chunk (16 values per thread, the three-round butterflies of rq_bfly_compact), its
+// codes staged in shared memory and stored as 32-bit words of four consecutive codes.
 // smem: kRQPartSmemBytes, 16-byte aligned; 256 threads meet at sync(); the caller
 // synchronizes before reusing smem.
-template <int VPC, int MAXCH, class Sync>
-__device__ __forceinline__ void rotate_quant_row_part_fast(const RQArgs& a, int row, int part, unsigned char* smem,
-                                                           int tid, Sync sync) {
-  static_assert(VPC == 4 || VPC == 8, "a part quantizes 4 or 8 values of each chunk per thread");
-  static_assert(VPC * MAXCH <= 16, "at most 16 kept values per thread");
-  constexpr int NP = 16 / VPC;
+template <class Sync>
+__device__ __forceinline__ void rotate_quant_part_blocks(const RQArgs& a, int row, int part, unsigned char* smem,
+                                                         int tid, Sync sync, long long wait_cycles, int* err) {
   long long* sx = reinterpret_cast<long long*>(smem);
-  uint8_t* stg = smem;   // [planes][K_pad] staged codes, in sx once its readers are done
-  float* redf = reinterpret_cast<float*>(smem + (size_t)kChunkPadded * 8 + 2 * kChunk);   // [8] warp maxima
+  uint8_t* stg = smem;   // staged codes [2][4096] (plane 1 at +4096), in sx once its readers are done
+  float* redf = reinterpret_cast<float*>(smem + (size_t)kChunkPadded * 8 + 2 * kChunk);
   unsigned long long* const tr = DPTQ_TRACE_BUF();
   (void)tr;
-  const int K = a.K;
-  const int K_pad = a.KB * 128;
-  const int tail_start = a.nfull << a.log2B;
-  const int bits = a.bits;
-  const int nch = (K + kChunk - 1) / kChunk;   // 1..MAXCH
-  const int e0 = part * VPC;                   // this part's values: e in [e0, e0 + VPC)
-  uint8_t* act = static_cast<uint8_t*>(a.out);
-  const size_t plane_stride = (size_t)a.KB * a.rows_out * 128;
-  auto store4 = [&](int k, uint32_t w0, uint32_t w1) {   // codes k .. k + 3 (k % 4 == 0)
-    const int kb = k >> 7, j = (k >> 4) & 7;
-    const size_t off = ((size_t)kb * a.rows_out + row) * 128 + ((j ^ (row & 7)) << 4) + (k & 15);
-    *reinterpret_cast<uint32_t*>(act + off) = w0;
-    if (bits == 8) *reinterpret_cast<uint32_t*>(act + plane_stride + off) = w1;
-  };
-
-  if (row >= a.rows_in) {   // padding row: zero codes (words split evenly over the parts) and scale
-    const int W = K_pad / 4;
-    for (int w = W * part / NP + tid; w < W * (part + 1) / NP; w += kRQThreads) store4(4 * w, 0u, 0u);
-    if (part == 0 && tid == 0 && a.scales != nullptr) a.scales[row] = 0.f;
+  if (row >= a.rows_in) {
+    part_zero_row(a, row, part, tid);
     return;
   }
   if (tid == 0) DPTQ_TRACE_CLOCK(tr, 170);
-  const uint4* src = reinterpret_cast<const uint4*>(a.x + (size_t)row * K);
-  float kept[MAXCH][VPC];
-  int kept_L = 0;   // layout of every chunk (the same for all chunks of a row but a shorter last one)
-  int last_L = 0;
-  long long mB = 0, mT = 0;
-  uint4 u[2];
-  rq_load16(src, 0, min(kChunk, K), tid, u);
-#pragma unroll 1
-  for (int c = 0; c < nch; ++c) {
-    const int c0 = c * kChunk;
-    const int len = min(kChunk, K - c0);
-    long long f[16];
+  const int K = a.K;
+  const int tail_start = a.nfull << a.log2B;
+  const int gr = a.B > 128 ? a.B : 128;
+  int g0, g1;
+  part_granules((K + gr - 1) / gr, a.np, part, g0, g1);
+  const int c0 = min(K, g0 * gr);
+  const int len = min(K, g1 * gr) - c0;   // 0 .. 4096, a multiple of 32
+  long long f[16];
+  {
+    uint4 u[2];
+    rq_load16(reinterpret_cast<const uint4*>(a.x + (size_t)row * K), c0, len, tid, u);
     rq_fix16(a, u, c0, len, tid, f);
-    if (c + 1 < nch) rq_load16(src, c0 + kChunk, min(kChunk, K - c0 - kChunk), tid, u);
-    if (tid == 0 && c == 0) DPTQ_TRACE_CLOCK(tr, 171);
-    const int L = rq_bfly_compact(a, c0, len, tail_start, f, sx, tid, sync);
-    if (tid == 0 && c == 0) DPTQ_TRACE_CLOCK(tr, 176);
-    if (c == 0) kept_L = L;
-    last_L = L;
-    if (len == kChunk && c0 + len <= tail_start) {   // every value is in a block of size B
-      long long m[8];   // pairwise tree: four dependent steps instead of sixteen
+  }
+  if (tid == 0) DPTQ_TRACE_CLOCK(tr, 171);
+  const int L = len > 0 ? rq_bfly_compact(a, c0, len, tail_start, f, sx, tid, sync) : 2;
+  if (tid == 0) DPTQ_TRACE_CLOCK(tr, 176);
+  // Block size of the part's values: one size unless the part reaches into the tail
+  // block from a whole block.  Values past len are zero (whole zero blocks).
+  const bool mixed = c0 < tail_start && c0 + len > tail_start;
+  const int lgp = c0 >= tail_start ? a.log2T : a.log2B;
+  float tmax;
+  if (!mixed) {
+    long long m[8];   // pairwise tree of |S|
 #pragma unroll
-      for (int e = 0; e < 8; ++e) {
-        const long long p = f[e] < 0 ? -f[e] : f[e], q = f[e + 8] < 0 ? -f[e + 8] : f[e + 8];
-        m[e] = p > q ? p : q;
-      }
-#pragma unroll
-      for (int w = 4; w > 0; w >>= 1)
-#pragma unroll
-        for (int e = 0; e < w; ++e) m[e] = m[e] > m[e + w] ? m[e] : m[e + w];
-      mB = m[0] > mB ? m[0] : mB;
-    } else {
-#pragma unroll
-      for (int e = 0; e < 16; ++e) {
-        const int i = rq_pos(L, tid, e);
-        const long long v = f[e] < 0 ? -f[e] : f[e];
-        if (i < len) {
-          if (c0 + i < tail_start)
-            mB = v > mB ? v : mB;
-          else
-            mT = v > mT ? v : mT;
-        }
-      }
-    }
-    long long v[VPC];   // f[e0 .. e0 + VPC - 1]; `part` is uniform over the CTA
-    if constexpr (VPC == 4) {
-      switch (part) {
-        case 0: v[0] = f[0]; v[1] = f[1]; v[2] = f[2]; v[3] = f[3]; break;
-        case 1: v[0] = f[4]; v[1] = f[5]; v[2] = f[6]; v[3] = f[7]; break;
-        case 2: v[0] = f[8]; v[1] = f[9]; v[2] = f[10]; v[3] = f[11]; break;
-        default: v[0] = f[12]; v[1] = f[13]; v[2] = f[14]; v[3] = f[15]; break;
-      }
-    } else {
-      if (part == 0) {
-#pragma unroll
-        for (int j = 0; j < 8; ++j) v[j] = f[j];
-      } else {
-#pragma unroll
-        for (int j = 0; j < 8; ++j) v[j] = f[8 + j];
-      }
-    }
-    float kv[VPC];
-#pragma unroll
-    for (int j = 0; j < VPC; ++j) {
-      const int i = rq_pos(L, tid, e0 + j);
-      kv[j] = i < len ? fixed_to_rotated(v[j], (c0 + i < tail_start) ? a.log2B : a.log2T, a.c_hi, a.c_lo) : 0.f;
+    for (int e = 0; e < 8; ++e) {
+      const long long p = f[e] < 0 ? -f[e] : f[e], q = f[e + 8] < 0 ? -f[e + 8] : f[e + 8];
+      m[e] = p > q ? p : q;
     }
 #pragma unroll
-    for (int cc = 0; cc < MAXCH; ++cc)   // kept[c] = kv with static register indices
-      if (cc == c) {
+    for (int w = 4; w > 0; w >>= 1)
 #pragma unroll
-        for (int j = 0; j < VPC; ++j) kept[cc][j] = kv[j];
-      }
+      for (int e = 0; e < w; ++e) m[e] = m[e] > m[e + w] ? m[e] : m[e + w];
+    tmax = m[0] ? fixed_to_rotated(m[0], lgp, a.c_hi, a.c_lo) : 0.f;
+  } else {
+    long long mB = 0, mT = 0;
+#pragma unroll
+    for (int e = 0; e < 16; ++e) {
+      const long long v = f[e] < 0 ? -f[e] : f[e];
+      if (c0 + rq_pos(L, tid, e) < tail_start)
+        mB = v > mB ? v : mB;
+      else
+        mT = v > mT ? v : mT;
+    }
+    tmax = fmaxf(mB ? fixed_to_rotated(mB, a.log2B, a.c_hi, a.c_lo) : 0.f,
+                 mT ? fixed_to_rotated(mT, a.log2T, a.c_hi, a.c_lo) : 0.f);
+  }
+  // The fp32 values, converted before the exchange so that their arithmetic overlaps it
+  // (the conversion is odd and monotone: the fp32 of the largest |S| is the largest |y|).
+  // This code runs once per launch from a cold instruction cache, so the uniform choices
+  // (one block size or two, even or odd log2) are taken once, outside the unrolled loops.
+  float y[16];
+  if (!mixed && (lgp & 1) == 0) {
+    const float sc = __int_as_float((127 - 24 - (lgp >> 1)) << 23);   // 2^-(24 + lgp / 2), exact
+#pragma unroll
+    for (int e = 0; e < 16; ++e) y[e] = __fmul_rn(ll_to_float_rn(f[e]), sc);
+  } else if (!mixed) {
+#pragma unroll
+    for (int e = 0; e < 16; ++e) y[e] = fixed_times_const(f[e], lgp >> 1, a.c_hi, a.c_lo);
+  } else {   // a part that reaches from a whole block into the tail block (rare)
+#pragma unroll
+    for (int e = 0; e < 16; ++e)
+      y[e] = fixed_to_rotated(f[e], (c0 + rq_pos(L, tid, e) < tail_start) ? a.log2B : a.log2T, a.c_hi, a.c_lo);
   }
   if (tid == 0) DPTQ_TRACE_CLOCK(tr, 140);
-  // Row absmax (see above); the barrier also ends every read of sx.
-  const float yB = mB ? fixed_to_rotated(mB, a.log2B, a.c_hi, a.c_lo) : 0.f;
-  const float yT = mT ? fixed_to_rotated(mT, a.log2T, a.c_hi, a.c_lo) : 0.f;
-  const uint32_t wmax = __reduce_max_sync(0xffffffffu, __float_as_uint(fmaxf(yB, yT)));
-  if ((tid & 31) == 0) redf[tid >> 5] = __uint_as_float(wmax);
-  sync();
-  float amax = redf[0];
-#pragma unroll
-  for (int w = 1; w < kRQThreads / 32; ++w) amax = fmaxf(amax, redf[w]);
-  const int qmax = (1 << (bits - 1)) - 1;
-  const float qmaxf = (float)qmax, qminf = (float)(-(1 << (bits - 1)));
+  const float amax = part_row_absmax(a, row, part, tmax, redf, tid, sync, wait_cycles, err);   // also ends sx's reads
+  if (tid == 0) DPTQ_TRACE_CLOCK(tr, 141);
+  const int bits = a.bits;
+  const float qmaxf = (float)((1 << (bits - 1)) - 1), qminf = -(float)(1 << (bits - 1));
   const float s = __fdiv_rn(amax, qmaxf);
   const bool nz = amax > 0.f;
   const float rs = nz ? __frcp_rn(s) : 0.f;
   if (part == 0 && tid == 0 && a.scales != nullptr) a.scales[row] = nz ? s : 0.f;
-  if (tid == 0) DPTQ_TRACE_CLOCK(tr, 141);
-
-  // Codes of this part, staged at their k (plane 0 at stg[k], plane 1 at stg[K_pad + k]).
-#pragma unroll 1
-  for (int c = 0; c < nch; ++c) {
-    const int c0 = c * kChunk;
-    const int len = min(kChunk, K - c0);
-    const int L = c + 1 < nch ? kept_L : last_L;
-    float kv[VPC];
+  // Codes into the staging bytes at their positions; A4 and A8 each in a loop of their own.
+  const int ib = L == 2 ? tid : L == 1 ? 256 * (tid >> 4) + (tid & 15) : 16 * tid;   // position of value 0
+  const int is = L == 2 ? 256 : L == 1 ? 16 : 1;                                       // and the stride
+  if (bits == 4) {
 #pragma unroll
-    for (int cc = 0; cc < MAXCH; ++cc)
-      if (cc == c) {
-#pragma unroll
-        for (int j = 0; j < VPC; ++j) kv[j] = kept[cc][j];
-      }
-#pragma unroll
-    for (int g4 = 0; g4 < VPC / 4; ++g4) {
-      float y[4] = {kv[4 * g4], kv[4 * g4 + 1], kv[4 * g4 + 2], kv[4 * g4 + 3]};
+    for (int g4 = 0; g4 < 4; ++g4) {
+      const float yy[4] = {y[4 * g4], y[4 * g4 + 1], y[4 * g4 + 2], y[4 * g4 + 3]};
       float q[4] = {0.f, 0.f, 0.f, 0.f};
-      if (nz) quant_code4(y, s, rs, qminf, qmaxf, q);
+      if (nz) quant_code4(yy, s, rs, qminf, qmaxf, q);
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
-        const int i = rq_pos(L, tid, e0 + 4 * g4 + j);
+        const int i = ib + is * (4 * g4 + j);
+        if (i < len) stg[i] = (uint8_t)e4m3_byte(q[j]);
+      }
+    }
+  } else {
+#pragma unroll
+    for (int g4 = 0; g4 < 4; ++g4) {
+      const float yy[4] = {y[4 * g4], y[4 * g4 + 1], y[4 * g4 + 2], y[4 * g4 + 3]};
+      float q[4] = {0.f, 0.f, 0.f, 0.f};
+      if (nz) quant_code4(yy, s, rs, qminf, qmaxf, q);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int i = ib + is * (4 * g4 + j);
         if (i < len) {
-          if (bits == 4) {
-            stg[c0 + i] = (uint8_t)e4m3_byte(q[j]);
-          } else {
-            const float m = fabsf(q[j]);
-            const float h = __fmul_rn(floorf(__fmul_rn(m, 0.0625f)), 16.f);
-            stg[c0 + i] = (uint8_t)e4m3_byte(__fadd_rn(copysignf(h, q[j]), 0.0f));
-            stg[K_pad + c0 + i] = (uint8_t)e4m3_byte(__fadd_rn(copysignf(__fsub_rn(m, h), q[j]), 0.0f));
-          }
+          uint32_t b0, b1;
+          part_code_bytes(q[j], 8, b0, b1);
+          stg[i] = (uint8_t)b0;
+          stg[kChunk + i] = (uint8_t)b1;
         }
       }
     }
   }
   if (tid == 0) DPTQ_TRACE_CLOCK(tr, 142);
   sync();
-  // The words whose values this part owns, VPC / 4 per thread and chunk, found directly
-  // from the layout: L = 2: k = 256 e + t, the part's values fill [256 e0, 256 (e0 + VPC));
-  // L = 1: k = 256 (t >> 4) + 16 e + (t & 15), the part's values fill 16 e0 .. 16 (e0 + VPC)
-  // within every 256-element block; L = 0: k = 16 t + e, the part's values are
-  // 16 t + e0 .. 16 t + e0 + VPC.
-  for (int c = 0; c < nch; ++c) {
-    const int c0 = c * kChunk;
-    const int len = min(kChunk, K - c0);
-    const int L = c + 1 < nch ? kept_L : last_L;
+  // Word j of this thread, found directly from the layout: L = 2 (value e at 256 e + t),
+  // L = 1 (256 (t >> 4) + 16 e + (t & 15)), L = 0 (16 t + e).
 #pragma unroll
-    for (int j = 0; j < VPC / 4; ++j) {
-      int i;
-      if (L == 2)
-        i = 256 * e0 + 4 * (j * kRQThreads + tid);
-      else if (L == 1)
-        i = 256 * (tid >> 4) + 16 * e0 + 4 * (j * 16 + (tid & 15));
-      else
-        i = 16 * tid + e0 + 4 * j;
-      if (i < len)
-        store4(c0 + i, *reinterpret_cast<const uint32_t*>(stg + c0 + i),
-               *reinterpret_cast<const uint32_t*>(stg + K_pad + c0 + i));
+  for (int j = 0; j < 4; ++j) {
+    const int i = L == 2 ? 4 * (j * kRQThreads + tid) : L == 1 ? 256 * (tid >> 4) + 4 * (j * 16 + (tid & 15)) : 16 * tid + 4 * j;
+    if (i < len)
+      part_store4(a, row, c0 + i, *reinterpret_cast<const uint32_t*>(stg + i),
+                  *reinterpret_cast<const uint32_t*>(stg + kChunk + i));
+  }
+  if (part == a.np - 1)   // k in [K, K_pad): zero codes
+    for (int k = K + 4 * tid; k < a.KB * 128; k += 4 * kRQThreads) part_store4(a, row, k, 0u, 0u);
+  if (tid == 0) DPTQ_TRACE_CLOCK(tr, 143);
+}
+
+// Block slices: output slice ps of block blk (B = n L, L = 256 V), thread t owning slice
+// positions V t .. V t + V - 1.  v = sum_a (-1)^popc(ps & a) x_a (exact), then the L-point
+// butterflies: log2 V levels in registers, 5 across the lanes (shuffles), 3 across the 8
+// warps (one exchange through shared memory, groups of 8 values on 32 V threads); the
+// codes go out as words without staging.  smem as rotate_quant_part_blocks.
+template <int V, class Sync>
+__device__ __forceinline__ void rotate_quant_part_slice(const RQArgs& a, int row, int part, unsigned char* smem,
+                                                        int tid, Sync sync, long long wait_cycles, int* err) {
+  static_assert(V == 4 || V == 8, "4 or 8 values per thread");
+  constexpr int L = 256 * V;
+  constexpr int U = L / 8;   // threads of the warp-level step
+  long long* sx = reinterpret_cast<long long*>(smem);   // [L], unpadded
+  float* redf = reinterpret_cast<float*>(smem + (size_t)kChunkPadded * 8 + 2 * kChunk);
+  unsigned long long* const tr = DPTQ_TRACE_BUF();
+  (void)tr;
+  if (row >= a.rows_in) {
+    part_zero_row(a, row, part, tid);
+    return;
+  }
+  if (tid == 0) DPTQ_TRACE_CLOCK(tr, 170);
+  const int n = a.B / L;   // parts per block: 2 or 4
+  const int ps = part % n;
+  const int k0 = (part / n) * a.B + V * tid;   // this thread's position in input slice 0
+  const __half* xr = a.x + (size_t)row * a.K + k0;
+  uint32_t raw[4][V / 2];   // the n slices' V fp16 values, all requested before any use
+#pragma unroll
+  for (int sl = 0; sl < 4; ++sl)
+    if (sl < n) {
+      if constexpr (V == 4) {
+        const uint2 w = *reinterpret_cast<const uint2*>(xr + sl * L);
+        raw[sl][0] = w.x;
+        raw[sl][1] = w.y;
+      } else {
+        const uint4 w = *reinterpret_cast<const uint4*>(xr + sl * L);
+        raw[sl][0] = w.x;
+        raw[sl][1] = w.y;
+        raw[sl][2] = w.z;
+        raw[sl][3] = w.w;
+      }
+    }
+  long long v[V];
+#pragma unroll
+  for (int i = 0; i < V; ++i) v[i] = 0;
+#pragma unroll
+  for (int sl = 0; sl < 4; ++sl)
+    if (sl < n) {
+      uint32_t sg = 0u;   // sign bits of the randomized Hadamard, one per value
+      if (a.signs != nullptr) {
+        const int8_t* sp = a.signs + k0 + sl * L;
+#pragma unroll
+        for (int i = 0; i < V; ++i) sg |= (sp[i] < 0 ? 1u : 0u) << i;
+      }
+      const bool neg = __popc(ps & sl) & 1;   // H_n[ps][sl] = -1
+#pragma unroll
+      for (int i = 0; i < V; ++i) {
+        long long t = half_to_fixed(i & 1 ? raw[sl][i >> 1] >> 16 : raw[sl][i >> 1] & 0xFFFFu);
+        if ((sg >> i) & 1u) t = -t;
+        v[i] = neg ? v[i] - t : v[i] + t;
+      }
+    }
+  if (tid == 0) DPTQ_TRACE_CLOCK(tr, 171);
+#pragma unroll
+  for (int h = 1; h < V; h <<= 1)
+#pragma unroll
+    for (int i = 0; i < V; ++i)
+      if ((i & h) == 0) {
+        const long long p = v[i], q = v[i + h];
+        v[i] = p + q;
+        v[i + h] = p - q;
+      }
+  const int lane = tid & 31;
+#pragma unroll
+  for (int b = 0; b < 5; ++b) {
+    const bool up = (lane >> b) & 1;   // the higher position of the pair
+#pragma unroll
+    for (int i = 0; i < V; ++i) {
+      const long long o = __shfl_xor_sync(0xffffffffu, v[i], 1 << b);
+      v[i] = up ? o - v[i] : v[i] + o;
     }
   }
-  if (part == NP - 1)   // k in [K, K_pad): zero codes
-    for (int k = K + 4 * tid; k < K_pad; k += 4 * kRQThreads) store4(k, 0u, 0u);
+#pragma unroll
+  for (int i = 0; i < V; i += 2) *reinterpret_cast<longlong2*>(sx + V * tid + i) = make_longlong2(v[i], v[i + 1]);
+  sync();
+  if (tid < U) {
+    long long w[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) w[k] = sx[tid + U * k];
+#pragma unroll
+    for (int h = 1; h < 8; h <<= 1)
+#pragma unroll
+      for (int k = 0; k < 8; ++k)
+        if ((k & h) == 0) {
+          const long long p = w[k], q = w[k + h];
+          w[k] = p + q;
+          w[k + h] = p - q;
+        }
+#pragma unroll
+    for (int k = 0; k < 8; ++k) sx[tid + U * k] = w[k];
+  }
+  sync();
+#pragma unroll
+  for (int i = 0; i < V; i += 2) {
+    const longlong2 t = *reinterpret_cast<const longlong2*>(sx + V * tid + i);
+    v[i] = t.x;
+    v[i + 1] = t.y;
+  }
+  if (tid == 0) DPTQ_TRACE_CLOCK(tr, 176);
+  long long mx = 0;
+#pragma unroll
+  for (int i = 0; i < V; ++i) {
+    const long long t = v[i] < 0 ? -v[i] : v[i];
+    mx = t > mx ? t : mx;
+  }
+  const float tmax = mx ? fixed_to_rotated(mx, a.log2B, a.c_hi, a.c_lo) : 0.f;
+  float y[V];   // exact 0 for S = 0; even or odd log2 B chosen once, outside the loop
+  if ((a.log2B & 1) == 0) {
+    const float sc = __int_as_float((127 - 24 - (a.log2B >> 1)) << 23);
+#pragma unroll
+    for (int i = 0; i < V; ++i) y[i] = __fmul_rn(ll_to_float_rn(v[i]), sc);
+  } else {
+#pragma unroll
+    for (int i = 0; i < V; ++i) y[i] = fixed_times_const(v[i], a.log2B >> 1, a.c_hi, a.c_lo);
+  }
+  if (tid == 0) DPTQ_TRACE_CLOCK(tr, 140);
+  const float amax = part_row_absmax(a, row, part, tmax, redf, tid, sync, wait_cycles, err);
+  if (tid == 0) DPTQ_TRACE_CLOCK(tr, 141);
+  const int bits = a.bits;
+  const float qmaxf = (float)((1 << (bits - 1)) - 1), qminf = -(float)(1 << (bits - 1));
+  const float s = __fdiv_rn(amax, qmaxf);
+  const bool nz = amax > 0.f;
+  const float rs = nz ? __frcp_rn(s) : 0.f;
+  if (part == 0 && tid == 0 && a.scales != nullptr) a.scales[row] = nz ? s : 0.f;
+  const int kout = (part / n) * a.B + ps * L + V * tid;   // first output position of this thread
+#pragma unroll
+  for (int g4 = 0; g4 < V / 4; ++g4) {
+    const float yy[4] = {y[4 * g4], y[4 * g4 + 1], y[4 * g4 + 2], y[4 * g4 + 3]};
+    float q[4] = {0.f, 0.f, 0.f, 0.f};
+    if (nz) quant_code4(yy, s, rs, qminf, qmaxf, q);
+    uint32_t w0 = 0u, w1 = 0u;
+    if (bits == 4) {
+#pragma unroll
+      for (int j = 0; j < 4; ++j) w0 |= e4m3_byte(q[j]) << (8 * j);
+    } else {
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        uint32_t b0, b1;
+        part_code_bytes(q[j], 8, b0, b1);
+        w0 |= b0 << (8 * j);
+        w1 |= b1 << (8 * j);
+      }
+    }
+    part_store4(a, row, kout + 4 * g4, w0, w1);
+  }
   if (tid == 0) DPTQ_TRACE_CLOCK(tr, 143);
 }
 

@@ -334,6 +334,52 @@ def test_fused_qlinear_equals_two_launches(dp, M, N, K, B):
     layer.close()
 
 
+# How the fused launch splits each row over its parts (np per row, from the planner):
+# slices of one block (1024 or 2048 elements per part) when a row has fewer blocks than
+# parts, else whole 128-aligned groups of blocks per part.
+FUSED_SPLIT_CASES = [
+    (5, 4096, 4096, 4096, False, 4),     # slices of 1024, four per block
+    (8, 4096, 4096, 2048, True, 4),      # slices of 1024, two per block; randomized signs
+    (64, 4096, 4096, 4096, False, 2),    # slices of 2048, two per block
+    (32, 12288, 4096, 4096, True, 2),    # q|k|v at M = 32 (96 CTAs): slices of 2048; signs
+    (64, 4096, 8192, 256, True, 2),      # whole blocks, two parts of 4096; signs
+    (64, 4096, 11008, 256, False, 4),    # whole blocks, four parts, two rounds of rows
+    (32, 4096, 14336, 2048, False, 4),   # whole blocks of 2048: 1 / 2 / 2 / 2 per part
+    (32, 4096, 6144, 4096, True, 4),     # one block, the 2048 tail block, two empty parts
+    (4, 4096, 224, 64, False, 2),        # a part holding a block of 64 and the 32-element tail
+    (16, 4096, 256, 256, False, 2),      # one part rotates the row, the other is empty
+]
+
+
+@pytest.mark.parametrize("M,N,K,B,rh,np_", FUSED_SPLIT_CASES)
+def test_fused_row_split_equals_two_launches(dp, M, N, K, B, rh, np_):
+    """Every row split of the fused launch (each part rotating only its own outputs, the
+    parts exchanging their maxima) gives the bits of the rotate-quantize launch and the
+    GEMM launch, which are compared with the oracle elsewhere."""
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    info = dp.dptq_plan_info(M, N, K, 4, sms, fused=True)
+    assert info["fused"] == 1 and info["rq_np"] == np_
+    wl = inputs.llama2_7b_decode()
+    x = torch.from_numpy(inputs.activations(wl, M, K)).to(DEV)
+    W = torch.from_numpy(inputs.weights(N, K, layer=5, proj=4)).to(DEV)
+    if rh:
+        d = np.where(np.random.default_rng(K + M).random(K) < 0.5, -1, 1).astype(np.int8)
+        layer = dp.dptq_pack_weights_rh(W, B, d)
+    else:
+        layer = dp.dptq_pack_weights(W, B)
+    for bits in (4, 8):
+        fused = torch.empty((M, N), dtype=torch.float16, device=DEV)
+        two = torch.empty((M, N), dtype=torch.float16, device=DEV)
+        for _ in range(3):   # repeated launches reuse the grid counters and the row-maximum slots
+            dp.dptq_qlinear(layer, x, bits, fused)
+        dp.dptq_qlinear_quantize(layer, x, bits)
+        dp.dptq_qlinear_gemm(layer, M, bits, two)
+        torch.cuda.synchronize()
+        assert torch.equal(fused.view(torch.int16), two.view(torch.int16)), (M, N, K, B, bits)
+    layer.close()
+    dp.dptq_last_device_error()
+
+
 def test_qlinear_m_zero_is_noop(dp):
     W = inputs.weights(128, 256)
     layer = dp.dptq_pack_weights(torch.from_numpy(W).to(DEV), 256)
