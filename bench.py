@@ -355,15 +355,24 @@ L2_BYTES = 129 * 2 ** 20
 
 
 def shape_cases():
-    """(label, M, N, K, had_block, bits): the LLaMA-2-7B decode projections and the
-    LLaMA-3-8B prefill ones (gate|up as one concatenated N)."""
+    """(label, M, N, K, had_block, bits): the LLaMA-2-7B decode projections, the
+    LLaMA-3-8B and LLaMA-2-13B prefill ones and the LLaMA-2-70B ones at four token counts
+    (q|k|v and gate|up as concatenated N), at A4 and, for the prefill shapes, A8."""
     d = [("7b qkv", 12288, 4096, 4096), ("7b o", 4096, 4096, 4096), ("7b gate|up", 22016, 4096, 4096),
          ("7b down", 4096, 11008, 256)]
     out = [(f"{n} decode", 32, N, K, B, 4) for n, N, K, B in d]
     out += [("7b gate|up decode", 32, 22016, 4096, 4096, 8), ("7b gate|up decode", 1, 22016, 4096, 4096, 4),
             ("7b gate|up decode", 8, 22016, 4096, 4096, 4)]
-    out += [("8b q prefill", 2048, 4096, 4096, 2048, 4), ("8b gate|up prefill", 2048, 28672, 4096, 2048, 4),
-            ("8b down prefill", 2048, 4096, 14336, 2048, 4)]
+    p8 = [("8b q prefill", 4096, 4096), ("8b gate|up prefill", 28672, 4096), ("8b down prefill", 4096, 14336)]
+    out += [(n, 2048, N, K, 2048, bits) for bits in (4, 8) for n, N, K in p8]
+    # LLaMA-2-13B prefill (M = 4096, block Hadamard 1024; gate|up A8 as on its masked layers)
+    p13 = [("13b qkv prefill", 15360, 5120), ("13b o prefill", 5120, 5120), ("13b gate|up prefill", 27648, 5120),
+           ("13b down prefill", 5120, 13824)]
+    out += [(n, 4096, N, K, 1024, 4) for n, N, K in p13] + [("13b gate|up prefill", 4096, 27648, 5120, 1024, 8)]
+    # LLaMA-2-70B (block Hadamard 4096) at M = 1, 64, 512 and 8192 tokens
+    p70 = [("70b qkv", 10240, 8192), ("70b o", 8192, 8192), ("70b gate|up", 57344, 8192), ("70b down", 8192, 28672)]
+    out += [(n, M, N, K, 4096, 4) for M in (1, 64, 512, 8192) for n, N, K in p70]
+    out += [("70b gate|up", 8192, 57344, 8192, 4096, 8)]
     return out
 
 

@@ -339,6 +339,16 @@ bool l2_prefetch_allowed() {
   return on;
 }
 
+// A8 prefill tiles: 192 tokens with the widened weights in tensor memory (default), or,
+// with DPTQ_A8_TILE128=1, 128 tokens with the weights widened into shared memory.
+bool a8_tile128() {
+  static const bool on = [] {
+    const char* v = std::getenv("DPTQ_A8_TILE128");
+    return v && v[0] == '1';
+  }();
+  return on;
+}
+
 // Weight stages a fused launch requests before its token rows are ready (DPTQ_PRE_STAGES,
 // a tuning knob; default 2).
 int pre_stages_setting() {

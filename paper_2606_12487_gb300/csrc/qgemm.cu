@@ -985,7 +985,7 @@ int gemm_pick_nt(int M, int bits, int KB) {
   if (M <= 16) return 16;
   if (M <= 32) return 32;
   if (M <= 64) return 64;
-  if (M <= 128 || bits == 8) return 128;
+  if (M <= 128 || (bits == 8 && a8_tile128())) return 128;
   return 192;
 }
 
@@ -1006,6 +1006,9 @@ bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan, i
   const int planes = bits == 8 ? 2 : 1;
   int nt = gemm_pick_nt(M, bits, KB);
   int kps = kps_for(nt);
+  // A8 192-token tiles take one k-block per stage: a stage holds two 24 KB activation
+  // planes, so two-block stages would leave room for only two of them.
+  if (nt == 192 && planes == 2) kps = 1;
   if (KB % kps != 0) kps = 1;
   // Largest |code| * |weight| sum per stage, and the stages one fp32 accumulator can
   // take before the exact-integer bound 2^24 could be crossed.
@@ -1020,8 +1023,9 @@ bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan, i
   seg_plan(kps, seg_iters, segs);
   while (nt > 16 && nt * segs > 512) {
     nt = nt == 192 ? 128 : nt >> 1;
-    if (kps_for(nt) != kps && KB % kps_for(nt) == 0) {
-      kps = kps_for(nt);
+    const int k2 = (nt == 192 && planes == 2) ? 1 : kps_for(nt);
+    if (k2 != kps && KB % k2 == 0) {
+      kps = k2;
       seg_plan(kps, seg_iters, segs);
     }
   }

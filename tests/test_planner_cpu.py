@@ -67,6 +67,9 @@ def test_split_plans_fit_and_cover(N, K, M, bits, sms):
     elif bits == 4 and M > 128:
         assert p["nt"] == 192 and p["a_tmem"] == 1
         assert p["kps"] == (2 if even_kb else 1)
+    elif bits == 8 and M > 128:
+        # two 24 KB activation planes per k-block: one k-block per stage, at least 4 stages
+        assert p["nt"] == 192 and p["a_tmem"] == 1 and p["kps"] == 1 and p["stages"] >= 4
     else:
         assert p["nt"] == 128 and p["kps"] == 1 and p["a_tmem"] == 0
 
