@@ -355,12 +355,14 @@ L2_BYTES = 129 * 2 ** 20
 
 
 def shape_cases():
-    """(label, M, N, K, had_block, bits): the LLaMA-2-7B decode projections, the
-    LLaMA-3-8B and LLaMA-2-13B prefill ones and the LLaMA-2-70B ones at four token counts
-    (q|k|v and gate|up as concatenated N), at A4 and, for the prefill shapes, A8."""
+    """(label, M, N, K, had_block, bits): the single 256 -> 512 linear, the LLaMA-2-7B
+    decode projections, the LLaMA-3-8B and LLaMA-2-13B prefill ones and the LLaMA-2-70B
+    ones at four token counts (q|k|v and gate|up as concatenated N), at A4 and, for the
+    prefill shapes, A8."""
     d = [("7b qkv", 12288, 4096, 4096), ("7b o", 4096, 4096, 4096), ("7b gate|up", 22016, 4096, 4096),
          ("7b down", 4096, 11008, 256)]
-    out = [(f"{n} decode", 32, N, K, B, 4) for n, N, K, B in d]
+    out = [("single linear 256->512", 16, 512, 256, 256, bits) for bits in (4, 8)]
+    out += [(f"{n} decode", 32, N, K, B, 4) for n, N, K, B in d]
     out += [("7b gate|up decode", 32, 22016, 4096, 4096, 8), ("7b gate|up decode", 1, 22016, 4096, 4096, 4),
             ("7b gate|up decode", 8, 22016, 4096, 4096, 4)]
     p8 = [("8b q prefill", 4096, 4096), ("8b gate|up prefill", 28672, 4096), ("8b down prefill", 4096, 14336)]
