@@ -339,6 +339,16 @@ bool l2_prefetch_allowed() {
   return on;
 }
 
+// Decode grids of one CTA per whole weight tile when the tiles fit the SMs (default), or,
+// with DPTQ_DECODE_WHOLE_TILES=0, every SM with split tiles (tuning).
+bool decode_whole_tiles() {
+  static const bool on = [] {
+    const char* v = std::getenv("DPTQ_DECODE_WHOLE_TILES");
+    return !(v && v[0] == '0');
+  }();
+  return on;
+}
+
 // A8 prefill tiles: 192 tokens with the widened weights in tensor memory (default), or,
 // with DPTQ_A8_TILE128=1, 128 tokens with the weights widened into shared memory.
 bool a8_tile128() {

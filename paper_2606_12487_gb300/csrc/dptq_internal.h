@@ -186,6 +186,7 @@ int take_rows_shortfall();
 // Decode GEMM launches prefetch their weight share into L2 unless DPTQ_L2PF=0.
 bool l2_prefetch_allowed();
 int pre_stages_setting();
+bool decode_whole_tiles();   // DPTQ_DECODE_WHOLE_TILES=0: decode grids never shrink to one CTA per tile
 bool a8_tile128();   // DPTQ_A8_TILE128=1: A8 prefill on 128-token tiles (weights widened into shared memory)
 // The GEMM operand rows are rotated and quantized by the whole-row kernel (sums kept in
 // registers) unless DPTQ_ROWS_KERNEL=0 (the per-row kernel with an fp32 row in shared

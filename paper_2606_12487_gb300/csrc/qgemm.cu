@@ -1074,8 +1074,11 @@ bool plan_gemm(int M, int N, int K_pad, int bits, int num_sms, GemmPlan& plan, i
     // extra round trip at the end of the launch; measured on GB300 that outweighs a
     // longer stream per CTA.  So: whole tiles, one per CTA, when they fit on the SMs and a
     // tile is at most twice a CTA's fair share of the stages; otherwise stream-K with at
-    // most four CTAs per tile.
-    if (tiles <= num_sms && (long long)KI * num_sms <= 2 * iters)
+    // most four CTAs per tile.  A fused launch keeps whole tiles only while they leave a
+    // CTA for each of four parts of every token row: with fewer, its rows would be split
+    // in two (slower rotation, measured: LLaMA-2-7B q|k|v at M = 32 is faster on all SMs).
+    const bool rows_fit = !fused || (long long)M_pad * 4 <= tiles;
+    if (decode_whole_tiles() && rows_fit && tiles <= num_sms && (long long)KI * num_sms <= 2 * iters)
       G = (int)tiles;
     else if (4 * tiles < G)
       G = (int)(4 * tiles);

@@ -341,7 +341,8 @@ FUSED_SPLIT_CASES = [
     (5, 4096, 4096, 4096, False, 4),     # slices of 1024, four per block
     (8, 4096, 4096, 2048, True, 4),      # slices of 1024, two per block; randomized signs
     (64, 4096, 4096, 4096, False, 2),    # slices of 2048, two per block
-    (32, 12288, 4096, 4096, True, 2),    # q|k|v at M = 32 (96 CTAs): slices of 2048; signs
+    (32, 12288, 4096, 4096, True, 4),    # q|k|v at M = 32: all SMs (split tiles), slices of 1024; signs
+    (64, 12288, 4096, 4096, True, 2),    # q|k|v at M = 64: slices of 2048; signs
     (64, 4096, 8192, 256, True, 2),      # whole blocks, two parts of 4096; signs
     (64, 4096, 11008, 256, False, 4),    # whole blocks, four parts, two rounds of rows
     (32, 4096, 14336, 2048, False, 4),   # whole blocks of 2048: 1 / 2 / 2 / 2 per part

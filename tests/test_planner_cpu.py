@@ -88,13 +88,19 @@ def test_fused_decode_plans(N, K, M, bits):
             dptq.dptq_plan_info(M, N, K, bits, 152, fused=True)
         return
     split = dptq.dptq_plan_info(M, N, K, bits, 152)
-    M_pad, G = split["M_pad"], split["grid"]
-    if M_pad * 4 > 2 * G and (M_pad * 2 > G or K > 8192):
+    M_pad = split["M_pad"]
+    tiles = split["n_wtiles"] * split["m_tiles"]
+    # the largest grid a decode plan takes: every SM, at most four CTAs per weight tile
+    g_max = min(152, 4 * tiles, tiles * split["KI"])
+    if M_pad * 4 > 2 * g_max and (M_pad * 2 > g_max or K > 8192):
         # too few CTAs for the rows' parts: dptq_qlinear takes the two-launch path
         with pytest.raises(dptq.DptqError):
             dptq.dptq_plan_info(M, N, K, bits, 152, fused=True)
         return
     p = dptq.dptq_plan_info(M, N, K, bits, 152, fused=True)
+    # whole tiles (one CTA each) only when they leave a CTA for each of four parts per row
+    if p["grid"] == tiles and tiles < g_max:
+        assert M_pad * 4 <= tiles
     _check_plan(p, M, N, K, bits, 152)
     assert p["fused"] == 1 and p["kps"] == 2 and p["nt"] <= 64 and p["stages"] >= 3
     assert p["smem_bytes"] <= SMEM_LIMIT
