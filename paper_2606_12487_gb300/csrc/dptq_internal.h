@@ -134,7 +134,8 @@ struct GemmArgs {
   uint32_t tmem_cols;
   int out_vec;         // `out` is 16-byte aligned: the epilogue stores 8 channels at a time
   long long l2_prefetch;  // weight bytes past the first ring stages each CTA requests into L2 up front (0: none)
-  // Fused launch: weight stages the producer requests before the token rows are ready;
+  // Fused launch: weight stages the producer requests before the token rows are ready
+  // (set from pre_stages_setting());
   // the rest of the ring and the L2 prefetch wait for the rows (while the rows are
   // rotated, the parts' exchanges of their maxima cross the memory system, and a full
   // ring fill in flight delays them by microseconds).
