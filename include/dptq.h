@@ -170,10 +170,12 @@ dptq_status dptq_sensitivity_policy(const float* x, const float* dx, int L, int 
  * at least twice larger buffers and keeps the superseded ones allocated until the process
  * exits, so work enqueued earlier and graphs captured earlier (which keep the old
  * addresses) stay valid.
- * For token tiles of up to 64 rows (M <= 64) whose rotation fits next to the GEMM's
- * pipeline in one CTA's shared memory, rotation, quantization and GEMM run as ONE
- * kernel launch (the environment variable DPTQ_FUSED=0 selects the two-launch
- * sequence of dptq_qlinear_quantize + dptq_qlinear_gemm); both give the same bits. */
+ * For token tiles of up to 64 rows (M <= 64), K <= 16384 and a power-of-two tail block,
+ * rotation, quantization and GEMM run as ONE kernel launch: each token row is split over
+ * two or four CTAs of the GEMM grid, each rotating and quantizing its own share of the
+ * row, and the row maxima are exchanged between them (the environment variable
+ * DPTQ_FUSED=0 selects the two-launch sequence of dptq_qlinear_quantize +
+ * dptq_qlinear_gemm); both give the same bits. */
 dptq_status dptq_qlinear(dptq_handle h, const void* x_fp16, int M, int bits, void* out_fp16,
                          void* stream);
 
