@@ -17,10 +17,18 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 OUT_DIR = os.path.join(HERE, "_build")
 LIB = os.path.join(OUT_DIR, "libdptq.so")
-# DPTQ_TRACE=1 builds a separate library whose kernels record %globaltimer stamps.
+# DPTQ_TRACE=1 builds a separate library whose kernels record %globaltimer stamps;
+# DPTQ_DEBUG=1 one whose kernels check the index arithmetic of their global accesses
+# (DPTQ_CHECK in csrc/dptq_device.cuh).
 TRACE = os.environ.get("DPTQ_TRACE") == "1"
+DEBUG = os.environ.get("DPTQ_DEBUG") == "1"
+if TRACE and DEBUG:
+    raise RuntimeError("DPTQ_TRACE and DPTQ_DEBUG select different libraries: set one")
 if TRACE:
     OUT_DIR = os.path.join(HERE, "_build_trace")
+    LIB = os.path.join(OUT_DIR, "libdptq.so")
+if DEBUG:
+    OUT_DIR = os.path.join(HERE, "_build_debug")
     LIB = os.path.join(OUT_DIR, "libdptq.so")
 SOURCES = ["api.cu", "rotate_quant.cu", "qgemm.cu", "static_scratch.cu", "kv_policy.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
@@ -36,6 +44,7 @@ def nvcc() -> str:
 def _flags():
     return ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I", os.path.join(ROOT, "include"),
                    *(["-DDPTQ_TRACE"] if TRACE else []),
+                   *(["-DDPTQ_DEBUG"] if DEBUG else []),
                    *([f"-DDPTQ_TRACE_STAGES={int(os.environ['DPTQ_TRACE_STAGES'])}"]
                      if TRACE and os.environ.get("DPTQ_TRACE_STAGES") else []),
                    *(["-DDPTQ_TRACE_CLOCKS"] if TRACE and os.environ.get("DPTQ_TRACE_CLOCKS") == "1" else []),

@@ -16,6 +16,7 @@
 #include <vector>
 
 #include <cuda_runtime.h>
+#include <nvtx3/nvToolsExt.h>
 
 #include "../../include/dptq.h"
 #include "dptq_internal.h"
@@ -323,6 +324,27 @@ bool pdl_allowed() {
   return on;
 }
 
+// NVTX ranges named after the entry points, around every call that launches work, for
+// timelines in NVIDIA's tools (DPTQ_NVTX=1; off by default, when a range costs one load).
+bool nvtx_enabled() {
+  static const bool on = [] {
+    const char* v = std::getenv("DPTQ_NVTX");
+    return v && v[0] == '1';
+  }();
+  return on;
+}
+struct NvtxRange {
+  const bool on;
+  explicit NvtxRange(const char* name) : on(nvtx_enabled()) {
+    if (on) nvtxRangePushA(name);
+  }
+  ~NvtxRange() {
+    if (on) nvtxRangePop();
+  }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
+
 bool fused_allowed() {
   static const bool on = [] {
     const char* v = std::getenv("DPTQ_FUSED");
@@ -501,17 +523,20 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 }  // namespace
 
 dptq_status dptq_pack_weights(const void* W_fp16, int N, int K, int had_block, int w_on_device, dptq_handle* out) {
+  NvtxRange nvtx_range("dptq_pack_weights");
   return pack_weights_impl(W_fp16, N, K, had_block, nullptr, w_on_device, out);
 }
 
 dptq_status dptq_pack_weights_rh(const void* W_fp16, int N, int K, int had_block, const int8_t* signs_host,
                                  int w_on_device, dptq_handle* out) {
+  NvtxRange nvtx_range("dptq_pack_weights_rh");
   if (!signs_host) return fail(DPTQ_ERR_INVALID_ARG, "null pointer");
   return pack_weights_impl(W_fp16, N, K, had_block, signs_host, w_on_device, out);
 }
 
 dptq_status dptq_rotate_quant_act_rh(const void* x_fp16, int M, int K, int had_block, int bits,
                                      const int8_t* signs_dev, void* codes, float* scales, void* stream) {
+  NvtxRange nvtx_range("dptq_rotate_quant_act_rh");
   if (bits != 4 && bits != 8) return fail(DPTQ_ERR_INVALID_ARG, "bits must be 4 or 8");
   if (M < 0 || K <= 0 || had_block <= 0) return fail(DPTQ_ERR_INVALID_ARG, "bad sizes");
   if (M == 0) return DPTQ_OK;
@@ -529,6 +554,7 @@ dptq_status dptq_rotate_quant_act_rh(const void* x_fp16, int M, int K, int had_b
 
 dptq_status dptq_rotate_act_rh(const void* x_fp16, int M, int K, int had_block, const int8_t* signs_dev,
                                float* y_f32, void* stream) {
+  NvtxRange nvtx_range("dptq_rotate_act_rh");
   if (M < 0 || K <= 0 || had_block <= 0) return fail(DPTQ_ERR_INVALID_ARG, "bad sizes");
   if (M == 0) return DPTQ_OK;
   if (!x_fp16 || !y_f32) return fail(DPTQ_ERR_INVALID_ARG, "null pointer");
@@ -545,6 +571,7 @@ dptq_status dptq_rotate_act_rh(const void* x_fp16, int M, int K, int had_block, 
 
 dptq_status dptq_rotate_quant_act(const void* x_fp16, int M, int K, int had_block, int bits, void* codes,
                                   float* scales, void* stream) {
+  NvtxRange nvtx_range("dptq_rotate_quant_act");
   if (bits != 4 && bits != 8) return fail(DPTQ_ERR_INVALID_ARG, "bits must be 4 or 8");
   if (M < 0 || K <= 0 || had_block <= 0) return fail(DPTQ_ERR_INVALID_ARG, "bad sizes");
   if (M == 0) return DPTQ_OK;
@@ -559,6 +586,7 @@ dptq_status dptq_rotate_quant_act(const void* x_fp16, int M, int K, int had_bloc
 }
 
 dptq_status dptq_rotate_act(const void* x_fp16, int M, int K, int had_block, float* y_f32, void* stream) {
+  NvtxRange nvtx_range("dptq_rotate_act");
   if (M < 0 || K <= 0 || had_block <= 0) return fail(DPTQ_ERR_INVALID_ARG, "bad sizes");
   if (M == 0) return DPTQ_OK;
   if (!x_fp16 || !y_f32) return fail(DPTQ_ERR_INVALID_ARG, "null pointer");
@@ -605,6 +633,7 @@ dptq_status quantize_into_scratch(dptq_handle h, const void* x_fp16, int M, int 
 extern "C" {
 
 dptq_status dptq_qlinear(dptq_handle h, const void* x_fp16, int M, int bits, void* out_fp16, void* stream) {
+  NvtxRange nvtx_range("dptq_qlinear");
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   int dev;
   GemmPlan plan;
@@ -630,6 +659,7 @@ dptq_status dptq_qlinear(dptq_handle h, const void* x_fp16, int M, int bits, voi
 }
 
 dptq_status dptq_qlinear_quantize(dptq_handle h, const void* x_fp16, int M, int bits, void* stream) {
+  NvtxRange nvtx_range("dptq_qlinear_quantize");
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   int dev;
   GemmPlan plan;
@@ -641,6 +671,7 @@ dptq_status dptq_qlinear_quantize(dptq_handle h, const void* x_fp16, int M, int 
 }
 
 dptq_status dptq_qlinear_gemm(dptq_handle h, int M, int bits, void* out_fp16, void* stream) {
+  NvtxRange nvtx_range("dptq_qlinear_gemm");
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   int dev;
   GemmPlan plan;
@@ -653,6 +684,7 @@ dptq_status dptq_qlinear_gemm(dptq_handle h, int M, int bits, void* out_fp16, vo
 
 dptq_status dptq_qgemm_codes(dptq_handle h, const void* codes, const float* scales, int M, int bits, void* out_fp16,
                              int32_t* acc_i32, void* stream) {
+  NvtxRange nvtx_range("dptq_qgemm_codes");
   if (bits != 4 && bits != 8) return fail(DPTQ_ERR_INVALID_ARG, "bits must be 4 or 8");
   if (M < 0) return fail(DPTQ_ERR_INVALID_ARG, "M must be >= 0");
   int dev;
@@ -681,6 +713,7 @@ dptq_status dptq_qgemm_codes(dptq_handle h, const void* codes, const float* scal
 
 dptq_status dptq_kv4_quantize(const void* kv_fp16, int rows, int cols, int group, void* codes, float* scales,
                               void* stream) {
+  NvtxRange nvtx_range("dptq_kv4_quantize");
   if (rows < 0 || cols <= 0 || group <= 0) return fail(DPTQ_ERR_INVALID_ARG, "bad sizes");
   if (rows == 0) return DPTQ_OK;
   if (!kv_fp16 || !codes || !scales) return fail(DPTQ_ERR_INVALID_ARG, "null pointer");
@@ -700,6 +733,7 @@ dptq_status dptq_kv4_quantize(const void* kv_fp16, int rows, int cols, int group
 dptq_status dptq_sensitivity_policy(const float* x, const float* dx, int L, int T, int d, int bits, double eps,
                                     double tau_jr, double tau_snr, double* jr, double* snr, uint8_t* bits_out,
                                     void* stream) {
+  NvtxRange nvtx_range("dptq_sensitivity_policy");
   if (bits != 4 && bits != 8) return fail(DPTQ_ERR_INVALID_ARG, "bits must be 4 or 8");
   if (L < 0 || T <= 0 || d <= 0 || !(eps >= 0.0)) return fail(DPTQ_ERR_INVALID_ARG, "bad sizes or eps");
   if (L == 0) return DPTQ_OK;
@@ -735,6 +769,7 @@ dptq_status dptq_plan_info(int M, int N, int K, int bits, int num_sms, int fused
 }
 
 dptq_status dptq_reserve(int max_M, int max_K, int max_N) {
+  NvtxRange nvtx_range("dptq_reserve");
   if (max_M < 0 || max_K < 0 || max_N < 0) return fail(DPTQ_ERR_INVALID_ARG, "sizes must be >= 0");
   int dev;
   dptq_status st = current_device(&dev);

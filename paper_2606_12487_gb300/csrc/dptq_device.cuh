@@ -79,6 +79,20 @@ enum DeviceError : int {
   kDevTimeoutRowMax = 0x108,   // a row's parts did not all post their maxima
 };
 
+// ------------------------------------------------------------------ debug checks
+// Built with -DDPTQ_DEBUG (a separate library, see build.py), DPTQ_CHECK(cond, err, site)
+// tests the index arithmetic of a global access: when cond is false it records
+// kDevBoundsCheck + site in the error word (the first failure wins) and evaluates to
+// false, so that the caller skips the access.  Otherwise it is the constant true and the
+// check compiles to nothing.  No check traps.
+constexpr int kDevBoundsCheck = 0x200;
+#ifdef DPTQ_DEBUG
+#define DPTQ_CHECK(cond, err, site) \
+  ((cond) ? true : (atomicCAS((err), 0, ::dptq::kDevBoundsCheck + (site)), false))
+#else
+#define DPTQ_CHECK(cond, err, site) true
+#endif
+
 // About one second at the GB300's ~2 GHz SM clock: any single wait longer than this
 // means the pipeline is broken, so the kernel records an error and unwinds instead of
 // spinning forever.

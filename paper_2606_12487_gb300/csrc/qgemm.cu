@@ -365,12 +365,18 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
           if (wprod) {
             if (g < kTraceStages) DPTQ_TRACE_POINT(tr, 8 + g);
             mbar_arrive_expect_tx(&full[s], w_bytes);
-            bulk_g2s(sm.wpack(s), wsrc, w_bytes, &full[s], pol_w);
+            // debug builds: the stage's weight bytes lie inside the packed tiles (site 1)
+            if (DPTQ_CHECK(nt < a.n_wtiles && (it + 1) * KPS <= a.KB, a.err, 1))
+              bulk_g2s(sm.wpack(s), wsrc, w_bytes, &full[s], pol_w);
             if (g < kTraceStages) DPTQ_TRACE_POINT(tr, 24 + g);
             if (g == S - 1) prefetch_share();
           } else {
             mbar_arrive_expect_tx(&afull[s], a_tx);
-            if (kb_stride == act_bytes) {
+            // debug builds: the stage's token tile lies inside the operand planes (site 2)
+            if (!DPTQ_CHECK(mt < a.m_tiles && (it + 1) * KPS <= a.KB, a.err, 2)) {
+              // skipped: the stage's barrier never completes, and the consumers' bounded
+              // waits end the launch with the check's code already in the error word
+            } else if (kb_stride == act_bytes) {
               // One token tile: a plane's KPS k-blocks are contiguous in global memory and in
               // the stage, so each plane is one copy (the bulk-copy engine's cost is largely
               // per copy).
@@ -735,7 +741,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1) qgemm_kernel(const GemmArgs a
       tc_fence_after();
       const int nseg = (un.i1 - 1) / a.seg_iters - un.i0 / a.seg_iters + 1;
       const uint32_t tb = tmem_base + lane_base + (uint32_t)(b * NT * a.segs);
-      int32_t* __restrict__ wsl = un.slot >= 0 ? ws_g + (size_t)un.slot * (NT * 128) : nullptr;
+      // debug builds: a split tile's slot is one of the grid's (site 3)
+      int32_t* __restrict__ wsl =
+          un.slot >= 0 && DPTQ_CHECK(un.slot < (int)gridDim.x, a.err, 3) ? ws_g + (size_t)un.slot * (NT * 128) : nullptr;
       // Split tile.  If every other contributor has already added its part to the slot,
       // this CTA finishes the tile straight from its accumulators (slot + own part);
       // otherwise it adds its part and the last contributor to arrive finishes.

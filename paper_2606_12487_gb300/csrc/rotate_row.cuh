@@ -803,7 +803,10 @@ __device__ __forceinline__ float part_row_absmax(const RQArgs& a, int row, int p
     float pm = redf[0];
 #pragma unroll
     for (int w = 1; w < kRQThreads / 32; ++w) pm = fmaxf(pm, redf[w]);
-    redf[8] = part_absmax_exchange(a.pmax + kRowMaxStride * row, a.np, part, pm, wait_cycles, err);
+    // debug builds: one of the 64 slot lines and a part of the row (site 6)
+    redf[8] = DPTQ_CHECK(row < 64 && part < a.np && a.np <= 4, err, 6)
+                  ? part_absmax_exchange(a.pmax + kRowMaxStride * row, a.np, part, pm, wait_cycles, err)
+                  : pm;
   }
   sync();
   return redf[8];
@@ -811,8 +814,10 @@ __device__ __forceinline__ float part_row_absmax(const RQArgs& a, int row, int p
 
 // Codes k .. k + 3 of `row` (k % 4 == 0) into the GEMM operand planes (the 128-byte
 // swizzled K-major layout of rotate_quant_row<kRQAct>).
-__device__ __forceinline__ void part_store4(const RQArgs& a, int row, int k, uint32_t w0, uint32_t w1) {
+__device__ __forceinline__ void part_store4(const RQArgs& a, int row, int k, uint32_t w0, uint32_t w1, int* err) {
   uint8_t* act = static_cast<uint8_t*>(a.out);
+  // debug builds: inside the operand planes (site 4)
+  if (!DPTQ_CHECK(row < a.rows_out && k >= 0 && k + 4 <= a.KB * 128 && (k & 3) == 0, err, 4)) return;
   const int kb = k >> 7, j = (k >> 4) & 7;
   const size_t off = ((size_t)kb * a.rows_out + row) * 128 + ((j ^ (row & 7)) << 4) + (k & 15);
   *reinterpret_cast<uint32_t*>(act + off) = w0;
@@ -821,9 +826,9 @@ __device__ __forceinline__ void part_store4(const RQArgs& a, int row, int k, uin
 
 // Padding row (row >= rows_in): zero codes, the K_pad / 4 words split evenly over the
 // parts, and a zero scale.
-__device__ __forceinline__ void part_zero_row(const RQArgs& a, int row, int part, int tid) {
+__device__ __forceinline__ void part_zero_row(const RQArgs& a, int row, int part, int tid, int* err) {
   const int W = a.KB * 32;
-  for (int w = W * part / a.np + tid; w < W * (part + 1) / a.np; w += kRQThreads) part_store4(a, row, 4 * w, 0u, 0u);
+  for (int w = W * part / a.np + tid; w < W * (part + 1) / a.np; w += kRQThreads) part_store4(a, row, 4 * w, 0u, 0u, err);
   if (part == 0 && tid == 0 && a.scales != nullptr) a.scales[row] = 0.f;
 }
 
@@ -854,7 +859,7 @@ __device__ __forceinline__ void rotate_quant_part_blocks(const RQArgs& a, int ro
   unsigned long long* const tr = DPTQ_TRACE_BUF();
   (void)tr;
   if (row >= a.rows_in) {
-    part_zero_row(a, row, part, tid);
+    part_zero_row(a, row, part, tid, err);
     return;
   }
   if (tid == 0) DPTQ_TRACE_CLOCK(tr, 170);
@@ -972,10 +977,10 @@ __device__ __forceinline__ void rotate_quant_part_blocks(const RQArgs& a, int ro
     const int i = L == 2 ? 4 * (j * kRQThreads + tid) : L == 1 ? 256 * (tid >> 4) + 4 * (j * 16 + (tid & 15)) : 16 * tid + 4 * j;
     if (i < len)
       part_store4(a, row, c0 + i, *reinterpret_cast<const uint32_t*>(stg + i),
-                  *reinterpret_cast<const uint32_t*>(stg + kChunk + i));
+                  *reinterpret_cast<const uint32_t*>(stg + kChunk + i), err);
   }
   if (part == a.np - 1)   // k in [K, K_pad): zero codes
-    for (int k = K + 4 * tid; k < a.KB * 128; k += 4 * kRQThreads) part_store4(a, row, k, 0u, 0u);
+    for (int k = K + 4 * tid; k < a.KB * 128; k += 4 * kRQThreads) part_store4(a, row, k, 0u, 0u, err);
   if (tid == 0) DPTQ_TRACE_CLOCK(tr, 143);
 }
 
@@ -995,14 +1000,16 @@ __device__ __forceinline__ void rotate_quant_part_slice(const RQArgs& a, int row
   unsigned long long* const tr = DPTQ_TRACE_BUF();
   (void)tr;
   if (row >= a.rows_in) {
-    part_zero_row(a, row, part, tid);
+    part_zero_row(a, row, part, tid, err);
     return;
   }
   if (tid == 0) DPTQ_TRACE_CLOCK(tr, 170);
   const int n = a.B / L;   // parts per block: 2 or 4
   const int ps = part % n;
   const int k0 = (part / n) * a.B + V * tid;   // this thread's position in input slice 0
-  const __half* xr = a.x + (size_t)row * a.K + k0;
+  // debug builds: the n slices lie inside the row (site 5); a failed check reads slice 0
+  const bool in_row = DPTQ_CHECK(k0 + (n - 1) * L + V <= a.K && n <= 4, err, 5);
+  const __half* xr = a.x + (size_t)row * a.K + (in_row ? k0 : 0);
   uint32_t raw[4][V / 2];   // the n slices' V fp16 values, all requested before any use
 #pragma unroll
   for (int sl = 0; sl < 4; ++sl)
@@ -1130,7 +1137,7 @@ __device__ __forceinline__ void rotate_quant_part_slice(const RQArgs& a, int row
         w1 |= b1 << (8 * j);
       }
     }
-    part_store4(a, row, kout + 4 * g4, w0, w1);
+    part_store4(a, row, kout + 4 * g4, w0, w1, err);
   }
   if (tid == 0) DPTQ_TRACE_CLOCK(tr, 143);
 }

@@ -3,6 +3,9 @@ function include/dptq.h declares, and rejects bad arguments before touching CUDA
 import ctypes
 import os
 import re
+import subprocess
+import sys
+import textwrap
 
 import pytest
 
@@ -105,3 +108,21 @@ def test_next_entry_points_check_arguments_without_gpu(lib):
     assert lib.dptq_sensitivity_policy(dummy, dummy, 2, 8, 63, 4, D(1e-6), D(0.1), D(20.0), dummy, dummy, dummy, None) == 1
     assert lib.dptq_sensitivity_policy(None, dummy, 2, 8, 64, 4, D(1e-6), D(0.1), D(20.0), dummy, dummy, dummy, None) == 1
     assert lib.dptq_sensitivity_policy(dummy, dummy, 0, 8, 64, 4, D(1e-6), D(0.1), D(20.0), dummy, dummy, dummy, None) == 0
+
+
+def test_nvtx_ranges_need_no_tool():
+    """With DPTQ_NVTX=1 every entry point opens and closes an NVTX range named after it;
+    with no profiler attached the calls behave as without (argument errors included)."""
+    code = textwrap.dedent("""
+        import ctypes
+        from paper_2606_12487_gb300 import dptq
+        lib = dptq.load()
+        d = ctypes.c_void_p(16)
+        print(lib.dptq_rotate_quant_act(d, 4, 256, 256, 5, d, d, None),
+              lib.dptq_rotate_quant_act(d, 4, 100, 64, 4, d, d, None),
+              lib.dptq_qlinear(None, d, 4, 4, d, None))
+    """)
+    env = dict(os.environ, DPTQ_NVTX="1")
+    r = subprocess.run([sys.executable, "-c", code], cwd=ROOT, env=env, capture_output=True, text=True, timeout=300)
+    assert r.returncode == 0, r.stdout + r.stderr
+    assert r.stdout.split() == ["1", "2", "1"]

@@ -154,3 +154,46 @@ def test_bounded_wait_times_out_and_recovers():
     line = r.stdout.strip().splitlines()[-1]
     assert line.startswith("5 0 same"), line
     assert "timed out" in line
+
+
+DEBUG_CHILD = """
+import hashlib
+import torch
+from paper_2606_12487_gb300 import dptq, inputs
+lib = dptq.load()
+dptq.dptq_reserve(192, 11008, 0)
+wl = inputs.llama2_7b_decode()
+h = hashlib.sha256()
+# fused: slices of 1024 (four parts), slices of 2048 (two parts), whole blocks; the two
+# launches at M = 5 and N = 384; a 192-token prefill tile at A4 and A8
+for M, N, K, B in [(32, 22016, 4096, 4096), (64, 4096, 4096, 4096), (32, 4096, 11008, 256), (5, 384, 11008, 256),
+                   (192, 1024, 4096, 2048)]:
+    W = torch.from_numpy(inputs.weights(N, K, layer=3, proj=1)).cuda()
+    layer = dptq.dptq_pack_weights(W, B)
+    x = torch.from_numpy(inputs.activations(wl, M, K)).cuda()
+    for bits in (4, 8):
+        out = torch.empty((M, N), dtype=torch.float16, device="cuda")
+        dptq.dptq_qlinear(layer, x, bits, out)
+        torch.cuda.synchronize()
+        h.update(out.cpu().numpy().tobytes())
+    layer.close()
+print(dptq.lib_path().split("/")[-2], lib.dptq_last_device_error(None), h.hexdigest())
+"""
+
+
+def test_debug_build_checks_pass_and_match_release():
+    """The DPTQ_DEBUG library checks the index arithmetic of the kernels' global accesses
+    (producers' tile copies, split-tile slots, the fused row parts' loads, stores and
+    maximum slots) and records the first failing check in the error word instead of
+    making the access.  On the fused, split and prefill paths no check fails, and the
+    outputs are the bits of the release library's."""
+    res = {}
+    for flag in ("0", "1"):
+        env = dict(os.environ, DPTQ_DEBUG=flag)
+        r = subprocess.run([sys.executable, "-c", textwrap.dedent(DEBUG_CHILD)], cwd=ROOT, env=env,
+                           capture_output=True, text=True, timeout=900)
+        assert r.returncode == 0, r.stdout + r.stderr
+        res[flag] = r.stdout.strip().splitlines()[-1].split()
+    assert res["1"][0] == "_build_debug" and res["0"][0] == "_build"
+    assert res["1"][1] == "0" and res["0"][1] == "0"
+    assert res["1"][2] == res["0"][2]
