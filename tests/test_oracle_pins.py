@@ -539,3 +539,25 @@ def test_fold_equivalence_with_paley_tail(orc):
     XR = np.array([orc.rotate_row_f64(x, B) for x in X])
     WR = np.array([orc.rotate_row_f64(w, B) for w in W])
     assert np.allclose(XR @ WR.T, X @ W.T, atol=1e-10)
+
+
+def test_randomized_hadamard_with_paley_tail(orc):
+    """QuaRot's randomized Hadamard D R (Sections 1 and 4.2) over a non-power-of-two tail
+    block: D R is still orthogonal (norms kept, Eq. 4), it equals the plain rotation of
+    x * d, it folds into the weights (Eq. 5), and the packed weights are the activation
+    quantizer applied to W with the same D R."""
+    K, B = 256 + 96, 256        # tail 96 = 12 x 8: H_12 (x) H_8
+    rng = np.random.default_rng(48)
+    d = _signs(K, 49)
+    x = inputs.to_f16(rng.standard_normal((3, K)).astype(np.float32))
+    W = inputs.to_f16((0.02 * rng.standard_normal((5, K))).astype(np.float32))
+    y = orc.rotate(x, B, signs=d).astype(np.float64)
+    xd = (x.astype(np.float64) * d).astype(np.float16)   # exact: a sign flip of binary16 values
+    assert np.array_equal(orc.rotate(xd, B), orc.rotate(x, B, signs=d))
+    xf, wf = x.astype(np.float64), W.astype(np.float64)
+    assert np.allclose(np.linalg.norm(y, axis=1), np.linalg.norm(xf, axis=1), rtol=1e-6)
+    yw = orc.rotate(W, B, signs=d).astype(np.float64)
+    assert np.allclose(y @ yw.T, xf @ wf.T, rtol=1e-5, atol=1e-6)
+    q, sw = orc.pack_weights(W, B, signs=d)
+    qc, sc = orc.rotate_quant_act(W, B, 4, signs=d)
+    assert np.array_equal(q, qc) and np.array_equal(sw, sc)
